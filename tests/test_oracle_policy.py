@@ -1,0 +1,265 @@
+"""Pins for the oracle's eviction policy and page layout (Sec. 3.3, "Online KV Eviction").
+
+Each pin comes from outside the oracle: hand-worked examples, an exhaustive
+enumeration of eviction sets that satisfy the wording of the rule, and the
+invariants the rule implies.
+"""
+import itertools
+import json
+import os
+
+import numpy as np
+import pytest
+
+from oracle.cache import OracleCache, OracleConfig
+from oracle.policy import SessionPolicy
+from synth.script import ACOUSTIC, ASR_DELIM, TEXT, TRANSCRIPT, UNIT_BEGIN
+
+EVICTABLE = {ACOUSTIC, ASR_DELIM}
+
+
+def _cache(budget, window, ps=4, n_pages=64, n_sessions=1):
+    return OracleCache(OracleConfig(n_sessions=n_sessions, layers=1, q_heads=1, kv_heads=1,
+                                    head_dim=4, page_size=ps, budget=budget, window=window,
+                                    dtype="f32", rope_base=10000.0, n_pages=n_pages))
+
+
+# -- hand-worked examples ----------------------------------------------------------------
+
+def _golden(golden_dir):
+    with open(os.path.join(golden_dir, "eviction_examples.json")) as f:
+        return json.load(f)["examples"]
+
+
+def test_hand_worked_examples(golden_dir):
+    for ex in _golden(golden_dir):
+        c = _cache(ex["budget"], ex["window"], ex["page_size"], ex["n_pages"])
+        if ex.get("prefix"):
+            c.append_chunk([0], [ex["prefix"]])
+        got = []
+        at_end = ex.get("evict_only_at_end", False)
+        for i, unit in enumerate(ex["units"]):
+            c.append_chunk([0], [unit])
+            if not at_end or i == len(ex["units"]) - 1:
+                before = set(c.policy[0].retained_positions())
+                res = c.evict([0])[0]
+                after = set(c.policy[0].retained_positions())
+                units = sorted({c.policy[0].unit[p] for p in before - after})
+                got.append({"resident": res, "evicted_units": units})
+        assert got == ex["after_each_evict"], ex["name"]
+        st = c.state(0)
+        fin = ex["final"]
+        assert st["pos"] == fin["retained"], ex["name"]
+        for key in ("hist_pages", "n_hist", "live_pages", "live_head", "n_live"):
+            assert st[key] == fin[key], (ex["name"], key)
+        assert sorted(c.pool._free) == fin["free_pages"], ex["name"]
+
+
+# -- brute force over every eviction set --------------------------------------------------
+
+def _brute_force_evicted_units(types, units, evicted, unit_cur, budget, window):
+    """Enumerate all sets of units; keep those that satisfy the rule's wording.
+
+    A set S of units is the rule's outcome when
+      (a) each member is eligible: 0 <= u <= unit_cur - W and holds a resident
+          evictable position;
+      (b) it is oldest-first: an eligible unit older than a member is a member;
+      (c) it stops correctly: after removing S, the count fits in B or no
+          eligible unit is left;
+      (d) it does not overshoot: before its newest member is removed, the count
+          still exceeded B.
+    """
+    n = len(types)
+
+    def resident_after(s):
+        return sum(1 for p in range(n) if not evicted[p]
+                   and not (units[p] in s and types[p] in EVICTABLE and units[p] >= 0))
+
+    eligible = sorted({units[p] for p in range(n) if not evicted[p] and units[p] >= 0
+                       and units[p] <= unit_cur - window and types[p] in EVICTABLE})
+    answers = []
+    for r in range(len(eligible) + 1):
+        for combo in itertools.combinations(eligible, r):
+            s = set(combo)
+            if any(u not in s and u < max(s, default=-10) for u in eligible):
+                continue
+            after = resident_after(s)
+            left = [u for u in eligible if u not in s]
+            if budget >= 0 and not (after <= budget or not left):
+                continue
+            if budget < 0 and s:
+                continue
+            if s:
+                prev = s - {max(s)}
+                if not resident_after(prev) > budget:
+                    continue
+            answers.append(s)
+    return answers
+
+
+def _random_script(rng, n_units, max_len):
+    tags = []
+    for _ in range(n_units):
+        k = int(rng.integers(1, max_len + 1))
+        body = [int(rng.choice([ACOUSTIC, ASR_DELIM, TRANSCRIPT, TEXT])) for _ in range(k)]
+        body[0] |= UNIT_BEGIN
+        tags.append(body)
+    return tags
+
+
+@pytest.mark.parametrize("seed", range(300))
+def test_brute_force_unique_choice(seed):
+    rng = np.random.default_rng(seed)
+    n_units = int(rng.integers(1, 5))
+    prefix = [int(rng.choice([ACOUSTIC, TEXT])) for _ in range(int(rng.integers(0, 3)))]
+    script = _random_script(rng, n_units, 6)
+    budget = int(rng.integers(-1, 12))
+    window = int(rng.integers(0, 4))
+    pol = SessionPolicy(budget, window)
+    pol.append(prefix)
+    evict_points = set(rng.choice(n_units, size=int(rng.integers(1, n_units + 1)),
+                                  replace=False).tolist()) | {n_units - 1}
+    for i, unit in enumerate(script):
+        pol.append(unit)
+        if i not in evict_points:
+            continue
+        before = list(pol.evicted)
+        answers = _brute_force_evicted_units(pol.type, pol.unit, before, pol.unit_cur,
+                                             budget, window)
+        assert len(answers) == 1, answers
+        got = pol.evict()
+        assert set(got) == answers[0]
+        assert got == sorted(got)
+
+
+# -- invariants of the rule ------------------------------------------------------------------
+
+def _run_random_session(seed, budget, window, n_units=40, evict_every=1):
+    rng = np.random.default_rng(seed)
+    pol = SessionPolicy(budget, window)
+    pol.append([TEXT] * int(rng.integers(0, 5)))
+    history = []
+    for u in range(n_units):
+        unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * int(rng.integers(0, 20))
+        if rng.random() < 0.8:
+            unit += [ASR_DELIM] + [TRANSCRIPT] * int(rng.poisson(3)) + [ASR_DELIM]
+        if rng.random() < 0.1:
+            unit += [TEXT] * int(rng.integers(1, 40))
+        pol.append(unit)
+        if u % evict_every == 0:
+            r_before = pol.resident()
+            was = list(pol.evicted)
+            evicted_units = pol.evict()
+            history.append((u, r_before, evicted_units, was))
+    return pol, history
+
+
+@pytest.mark.parametrize("budget,window", [(-1, 5), (0, 0), (0, 3), (50, 2), (100, 5),
+                                           (200, 10), (30, 0), (400, 1)])
+def test_policy_invariants(budget, window):
+    for seed in range(8):
+        pol, history = _run_random_session(seed, budget, window)
+        n = pol.pos_next
+        for p in range(n):
+            if pol.evicted[p]:
+                # (ii) only evictable positions of units >= 0 ever go
+                assert pol.unit[p] >= 0 and pol.type[p] in EVICTABLE
+        # (ii) transcripts, text and the prefix stay
+        for p in range(n):
+            if pol.type[p] in (TRANSCRIPT, TEXT) or pol.unit[p] < 0:
+                assert not pol.evicted[p]
+        # (ii) every position of the W most recent units stays
+        for p in range(n):
+            if pol.unit[p] > pol.unit_cur - window:
+                assert not pol.evicted[p]
+        # (i) after the last evict: fits, or nothing eligible remains
+        r = pol.resident()
+        if budget >= 0 and r > budget:
+            assert pol.oldest_eligible_unit() is None
+        # (iii) evicted units form a prefix of the units in age order
+        gone = sorted({pol.unit[p] for p in range(n) if pol.evicted[p]})
+        assert gone == list(range(len(gone)))
+        # (v) unbounded evicts nothing
+        if budget < 0:
+            assert not any(pol.evicted)
+        for _, r_before, evicted_units, _ in history:
+            assert evicted_units == sorted(evicted_units)
+
+
+def test_floor_budget_evicts_every_eligible_unit():
+    """B = 0 (Table 3's floor) leaves only protected positions and the window."""
+    for window in (0, 1, 5):
+        pol, _ = _run_random_session(3, 0, window)
+        for p in range(pol.pos_next):
+            eligible = 0 <= pol.unit[p] <= pol.unit_cur - window
+            assert pol.evicted[p] == (eligible and pol.type[p] in EVICTABLE)
+
+
+def test_budget_shape_like_table3():
+    """End <= B and Peak <= B + one unit's growth, on 17+segment units (Table 3 shape)."""
+    rng = np.random.default_rng(0)
+    # Unit counts chosen so that transcripts plus the window stay below B, as in
+    # the paper's sessions (End < B there); beyond that the stop rule applies.
+    for budget, n_units in ((512, 100), (1024, 250), (2048, 400)):
+        pol = SessionPolicy(budget, 5)
+        peak, max_growth = 0, 0
+        for u in range(n_units):
+            unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * 16 + [ASR_DELIM] + \
+                [TRANSCRIPT] * int(rng.poisson(3)) + [ASR_DELIM]
+            max_growth = max(max_growth, len(unit))
+            pol.append(unit)
+            peak = max(peak, pol.resident())
+            pol.evict()
+            assert pol.resident() <= budget
+        assert budget < peak <= budget + max_growth
+
+
+def test_mid_unit_evict_with_zero_window_keeps_scanning_current_unit():
+    """W = 0 lets the current unit go; tokens fed later to the same unit stay eligible."""
+    pol = SessionPolicy(0, 0)
+    pol.append([ACOUSTIC | UNIT_BEGIN, ACOUSTIC])
+    assert pol.evict() == [0]
+    pol.append([ACOUSTIC, TRANSCRIPT])
+    assert pol.evict() == [0]
+    assert pol.retained_positions() == [3]
+
+
+# -- layout contract -----------------------------------------------------------------------
+
+@pytest.mark.parametrize("seed", range(6))
+def test_layout_invariants_many_sessions(seed):
+    rng = np.random.default_rng(seed)
+    n_sessions, ps = 5, 4
+    c = _cache(int(rng.integers(5, 60)), int(rng.integers(0, 4)), ps=ps, n_pages=4000,
+               n_sessions=n_sessions)
+    total = c.pool.n_pages
+    for step in range(60):
+        active = sorted(rng.choice(n_sessions, size=int(rng.integers(1, n_sessions + 1)),
+                                   replace=False).tolist())
+        chunks = []
+        for s in active:
+            unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * int(rng.integers(0, 9))
+            unit += [ASR_DELIM] + [TRANSCRIPT] * int(rng.poisson(2)) + [ASR_DELIM]
+            chunks.append(unit)
+        c.append_chunk(active, chunks)
+        c.evict(active)
+        seen = set()
+        used = 0
+        for s in range(n_sessions):
+            st = c.state(s)
+            lay = c.layout[s]
+            # retained logical order is ascending position
+            assert st["pos"] == sorted(st["pos"])
+            # pages are exactly as many as the regions need
+            assert len(lay.hist_pages) == -(-lay.n_hist // ps)
+            assert len(lay.live_pages) == -(-(lay.live_head + lay.n_live) // ps)
+            assert 0 <= lay.live_head < ps
+            # no page appears twice, within or across sessions
+            for pid in lay.hist_pages + lay.live_pages:
+                assert pid not in seen
+                seen.add(pid)
+            used += len(lay.hist_pages) + len(lay.live_pages)
+            # every retained position has a distinct (page, slot)
+            slots = {lay.slot_of_logical(i) for i in range(len(st["pos"]))}
+            assert len(slots) == len(st["pos"])
+        assert used + c.pool.free_count() == total
