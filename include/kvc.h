@@ -1,0 +1,203 @@
+/*
+ * kvc.h - C interface of the GB300 library for acoustic-to-text KV eviction
+ * and retained-cache GQA attention ("Acoustic-to-Text KV Compression for
+ * Full-Duplex Speech Models", Sec. 3.1 and Sec. 3.3).
+ *
+ * The library keeps, per streaming session, a paged K/V cache for every
+ * layer.  Each fed position carries a type tag (acoustic, ASR delimiter,
+ * transcript, text).  kvc_evict applies the online eviction rule of
+ * Sec. 3.3: while the resident count exceeds the budget B, the acoustic and
+ * structural positions of the oldest unit outside the W most recent units
+ * are dropped; transcript, response text and the system prefix stay, and
+ * kept keys keep their original rotary positions.  The attention calls run
+ * over whatever is resident.
+ *
+ * Conventions for every call:
+ *  - Device memory (pool, metadata workspace, q/k/v/out, types) is owned by
+ *    the caller and must outlive the context.  The library never allocates
+ *    device memory.
+ *  - Calls taking a stream are asynchronous on it (cudaStream_t passed as
+ *    void*; NULL is the legacy default stream), except where a comment says
+ *    "synchronises".
+ *  - Arguments are validated on the host before any launch; on error the
+ *    call returns a negative status, launches nothing and changes no state.
+ *    kvc_last_error() then describes the failure (thread-local string).
+ *  - Kernels never trap.  A capacity check that can only fail on the device
+ *    records a code in a device error word and leaves the state as it was;
+ *    the next synchronising call returns KVC_EDEVICE (kvc_device_status
+ *    reports the recorded code).
+ *  - Layouts are row-major and contiguous.  The element type (binary32 or
+ *    bfloat16) is fixed at creation for K, V, q and out alike.
+ */
+#ifndef KVC_H
+#define KVC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct kvc_ctx kvc_ctx;
+
+/* Element types. */
+enum { KVC_F32 = 0, KVC_BF16 = 1 };
+
+/* Token type tags (low 7 bits of a type byte).  Sec. 3.3: ACOUSTIC (unit
+ * marker, audio tokens, native decision, terminators) and ASR_DELIM are
+ * evictable; TRANSCRIPT and TEXT (response text, system prefix) are kept. */
+enum { KVC_ACOUSTIC = 0, KVC_ASR_DELIM = 1, KVC_TRANSCRIPT = 2, KVC_TEXT = 3 };
+/* Flag on the first position of a duplex unit (Sec. 3.1); it opens a new
+ * unit.  Positions fed before the first flag belong to unit -1 (the system
+ * prefix) and are never evicted. */
+#define KVC_UNIT_BEGIN 0x80
+
+/* Status codes. */
+enum {
+  KVC_OK = 0,
+  KVC_EINVAL = -1,   /* bad argument */
+  KVC_ENOMEM = -2,   /* page pool or a capacity would overflow */
+  KVC_ECUDA = -3,    /* a CUDA runtime call failed */
+  KVC_ESTATE = -4,   /* call out of order (e.g. attention without append) */
+  KVC_EDEVICE = -5   /* a kernel recorded a failed check (kvc_device_status) */
+};
+
+/* Device error codes (bits of the device error word). */
+enum {
+  KVC_DERR_POOL = 1,         /* no free page where the host expected one */
+  KVC_DERR_PAGE_TABLE = 2,   /* a session's page list is full */
+  KVC_DERR_POSITION = 4,     /* position beyond max_positions */
+  KVC_DERR_MOVES = 8,        /* eviction move list full */
+  KVC_DERR_WAIT = 16         /* a pipeline wait gave up (bounded spin) */
+};
+
+typedef struct kvc_config {
+  int32_t n_sessions;            /* session ids are 0 .. n_sessions-1 */
+  int32_t layers;                /* L */
+  int32_t q_heads;               /* Hq */
+  int32_t kv_heads;              /* Hkv; Hq % Hkv == 0, G = Hq / Hkv */
+  int32_t head_dim;              /* D */
+  int32_t page_size;             /* positions per page; 16 */
+  int64_t budget;                /* B (Sec. 3.3); < 0 means unbounded */
+  int32_t window;                /* W >= 0 most recent units are never evicted */
+  int32_t dtype;                 /* KVC_F32 or KVC_BF16 */
+  double rope_base;              /* rotary base, e.g. 10000 */
+  int64_t n_pages;               /* pool capacity in pages */
+  int32_t max_pages_per_session; /* capacity of each of a session's two page lists */
+  int32_t max_positions;         /* positions fed to one session stay below this */
+  int32_t max_seq_per_call;      /* sessions per call, <= 512 */
+  int32_t max_tokens_per_call;   /* tokens per kvc_append_chunk call */
+} kvc_config;
+
+/* Supported shapes: (KVC_BF16, head_dim 128) and (KVC_F32, head_dim 64), with
+ * G = Hq / Hkv in {1, 2, 4, 8} and page_size 16. */
+
+typedef struct kvc_session_info {
+  int32_t pos_next;       /* next position id (= positions fed so far) */
+  int32_t unit_cur;       /* current unit, -1 before the first unit marker */
+  int32_t n_hist;         /* retained positions in the compacted (hist) region */
+  int32_t n_hist_pages;
+  int32_t live_head;      /* consumed slots at the front of the first live page */
+  int32_t n_live;         /* positions in the live region */
+  int32_t n_live_pages;
+  int32_t resident;       /* n_hist + n_live */
+  int32_t n_evicted;      /* positions evicted so far */
+  int32_t peak_resident;  /* largest resident count seen after an append */
+} kvc_session_info;
+
+/* Bytes of pool and metadata workspace a configuration needs.
+ * Pool layout: page-major, [n_pages][L][2 (K,V)][Hkv][page_size][D] elements.
+ * Returns KVC_EINVAL for unsupported or inconsistent configurations. */
+int kvc_query_sizes(const kvc_config* cfg, size_t* pool_bytes, size_t* meta_bytes);
+
+/* Create a context over caller-owned device memory (d_pool, d_meta, sizes
+ * from kvc_query_sizes or larger; 256-byte aligned).  Zeroes the pool,
+ * initialises the metadata and the rotary table (cos/sin of p * base^(-2i/D)
+ * evaluated in binary64, stored in binary32), then synchronises `stream`. */
+int kvc_create(kvc_ctx** out, const kvc_config* cfg, void* d_pool, size_t pool_bytes,
+               void* d_meta, size_t meta_bytes, void* stream);
+
+/* Free the host-side context.  Device memory stays the caller's. */
+void kvc_destroy(kvc_ctx* ctx);
+
+/* Feed tokens to sessions (one chunk per session): assign original position
+ * ids (Sec. 3.3: they advance with every fed token), open a unit at each
+ * KVC_UNIT_BEGIN, rotate K at its position (rotate-half RoPE) and write K, V
+ * and the {position, type, unit} tags at the live tail, allocating the lowest
+ * free pages in (call order, token order).
+ *   n_seq        number of sessions in the call, 1 .. max_seq_per_call
+ *   h_sessions   host [n_seq] distinct session ids
+ *   h_cu_tokens  host [n_seq+1] token offsets, h_cu_tokens[0] = 0, every
+ *                session gets >= 1 token; total <= max_tokens_per_call
+ *   d_types      device [total] type bytes
+ *   d_k, d_v     device [L][total][Hkv][D] un-rotated keys / values
+ * Returns KVC_ENOMEM (nothing launched) if the pool cannot hold the chunk.
+ * The chunk's queries are what the following attention calls answer. */
+int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions,
+                     const int32_t* h_cu_tokens, const uint8_t* d_types, const void* d_k,
+                     const void* d_v, void* stream);
+
+/* Online eviction (Sec. 3.3) for each listed session, run by the caller after
+ * a unit: while resident > B, evict the ACOUSTIC and ASR_DELIM positions of
+ * the oldest unit u with 0 <= u <= unit_cur - W that still has some; stop
+ * when resident <= B or no such unit remains.  Survivors of the consumed
+ * live prefix move (all layers, 16-byte copies) to the compacted region in
+ * position order; consumed live pages are freed.
+ *   d_resident_out  optional device [n_seq] int64: resident count afterwards
+ * Invalidates the last append's queries for attention. */
+int kvc_evict(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, int64_t* d_resident_out,
+              void* stream);
+
+/* Chunked-prefill GQA attention of one layer for the queries of the last
+ * appended chunk (e.g. the 17 acoustic positions of a unit): query t of a
+ * session sits at its position and sees every resident key at or before it
+ * (causal inside the chunk).  softmax(RoPE(q) . k / sqrt(D)) v, softmax in
+ * binary32, K/V products on tensor cores for bfloat16.
+ *   layer   0 .. L-1
+ *   d_q     device [total][Hq][D] un-rotated queries, total and order as in
+ *           the last kvc_append_chunk; chunks of at most 32 tokens
+ *   d_out   device [total][Hq][D]
+ * KVC_ESTATE if no append precedes it (or an evict/release came after). */
+int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out,
+                           void* stream);
+
+/* Single-token decode GQA attention of one layer (transcript, delimiter and
+ * response tokens): the last append gave each of its n_seq sessions exactly
+ * one token; that token attends to every resident key, itself included.
+ * Split-K over pages with a log-sum-exp merge.
+ *   d_q     device [n_seq][Hq][D] un-rotated queries (call order of the append)
+ *   d_out   device [n_seq][Hq][D] */
+int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void* stream);
+
+/* Resident count of one session (n_hist + n_live), including the system
+ * prefix and text (Sec. 3.3).  Synchronises the device. */
+int kvc_resident_size(kvc_ctx* ctx, int session, int64_t* h_out);
+
+/* End sessions: free all their pages and reset them to position 0. */
+int kvc_release(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, void* stream);
+
+/* Copy one session's state to host buffers (synchronises).  Page lists go to
+ * h_hist_pages / h_live_pages (capacity max_pages_per_session each); the
+ * resident positions' {position, type, unit} go, in retained order, to
+ * h_pos / h_type / h_unit (capacity `cap` entries each).  Any pointer but
+ * h_info may be NULL. */
+int kvc_export_state(kvc_ctx* ctx, int session, kvc_session_info* h_info,
+                     int32_t* h_hist_pages, int32_t* h_live_pages, int32_t* h_pos,
+                     uint8_t* h_type, int32_t* h_unit, int64_t cap);
+
+/* Copy the stored (rotated) K and V of one layer of one session, in retained
+ * order, to host buffers [cap][Hkv][D] each (synchronises). */
+int kvc_export_kv(kvc_ctx* ctx, int session, int layer, void* h_k, void* h_v, int64_t cap);
+
+/* Free pages in the pool and the device error word (synchronises). */
+int kvc_device_status(kvc_ctx* ctx, int64_t* h_free_pages, int32_t* h_error_bits);
+
+/* Description of the last failure on this thread ("" if none). */
+const char* kvc_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVC_H */

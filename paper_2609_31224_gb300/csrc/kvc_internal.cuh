@@ -1,0 +1,277 @@
+// Internal definitions of the kvc library: device state, metadata layout and
+// the PTX helpers (mbarrier, bulk copy) the kernels share.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/kvc.h"
+
+namespace kvc {
+
+constexpr int PS = 16;          // positions per page
+constexpr int MAX_SEQ = 512;    // sessions per call
+constexpr int TYPE_MASK = 0x7F;
+constexpr long long WAIT_LIMIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
+
+// Per-session device state.  The retained sequence is the hist region
+// (n_hist positions, densely packed from slot 0 of hist page 0) followed by
+// the live region (n_live positions from slot live_head of live page 0).
+struct SessState {
+  int32_t pos_next;
+  int32_t unit_cur;
+  int32_t n_hist;
+  int32_t n_hist_pages;
+  int32_t live_head;
+  int32_t n_live;
+  int32_t n_live_pages;
+  int32_t last_chunk;
+  int32_t n_evicted;
+  int32_t peak_resident;
+  int32_t pad[6];
+};
+static_assert(sizeof(SessState) == 64, "SessState size");
+
+// Snapshot of one session of the last append, read by the attention kernels.
+struct SeqInfo {
+  int32_t sid;
+  int32_t t;            // tokens in the chunk
+  int32_t q_row0;       // first query row of this session in q/out
+  int32_t pos_first;    // position of the chunk's first token
+  int32_t n_hist;
+  int32_t n_hist_pages;
+  int32_t live_head;
+  int32_t n_live;
+  int32_t n_blocks;     // n_hist_pages + n_live_pages
+  int32_t dec_chunks;   // split-K chunks of the decode work list
+  int32_t dec_base;     // first partial slot of this session (decode)
+  int32_t pf_chunks;
+  int32_t pf_base;
+  int32_t pad[3];
+};
+static_assert(sizeof(SeqInfo) == 64, "SeqInfo size");
+
+// One split-K work item: blocks [blk_begin, blk_end) of one session.
+struct Item {
+  int32_t seq;
+  int32_t chunk;
+  int32_t blk_begin;
+  int32_t blk_end;
+};
+
+struct DevGlobals {
+  int32_t err;
+  int32_t n_seq;
+  int64_t pages_used;
+  int32_t n_dec_items;
+  int32_t n_pf_items;
+  int32_t n_moves;
+  int32_t total_tokens;
+  int32_t pad[8];
+};
+
+// Device pointers into the caller's workspace plus the shape, passed by value.
+struct Dev {
+  // shape
+  int32_t n_sessions, layers, q_heads, kv_heads, head_dim, group;
+  int32_t esz;                 // bytes per element
+  int32_t max_pages_per_session, max_positions, max_seq, max_tokens;
+  int64_t budget;
+  int32_t window;
+  int64_t n_pages;
+  int32_t bitmap_words;
+  int32_t max_moves;
+  int32_t max_dec_items, max_pf_items;   // items including the kv-head factor
+  // memory
+  uint8_t* pool;
+  SessState* sess;
+  int32_t* hist_pt;            // [n_sessions][max_pages_per_session]
+  int32_t* live_pt;            // [n_sessions][max_pages_per_session]
+  int32_t* meta_pos;           // [n_pages * PS]
+  int32_t* meta_unit;          // [n_pages * PS]
+  uint8_t* meta_type;          // [n_pages * PS]
+  uint32_t* bitmap;            // 1 = page in use
+  DevGlobals* g;
+  float2* rope;                // [max_positions][D/2] (cos, sin)
+  SeqInfo* seq;                // [max_seq]
+  Item* dec_items;             // [max_dec_items]
+  Item* pf_items;              // [max_pf_items]
+  int32_t* tok_slot;           // [max_tokens] page * PS + slot
+  int32_t* tok_pos;            // [max_tokens]
+  int2* moves;                 // [max_moves] (src page*PS+slot, dst page*PS+slot)
+  int32_t* alloc_list;         // [max_alloc] pages handed out by the last allocation
+  int32_t max_alloc;
+  float* dec_part_o;           // [max_dec_items][G][D]
+  float2* dec_part_ml;         // [max_dec_items][G] (m, l) in log2 units
+  float* pf_part_o;            // [max_pf_items][PF_ROWS][D]
+  float2* pf_part_ml;          // [max_pf_items][PF_ROWS]
+  int32_t* dec_count;          // [max_seq * kv_heads] arrival counters
+  int32_t* pf_count;           // [max_seq * kv_heads]
+};
+
+constexpr int PF_MAX_TOKENS = 32;  // tokens per session per prefill call
+
+__host__ __device__ inline size_t pool_offset_elems(const Dev& d, int page, int layer, int kv,
+                                                    int head, int slot) {
+  return ((((size_t)page * d.layers + layer) * 2 + kv) * d.kv_heads + head) * (size_t)PS *
+             d.head_dim + (size_t)slot * d.head_dim;
+}
+
+// Page and valid slot range [lo, hi) of virtual block b of a session; the
+// logical (retained-order) index of slot s is base + s.
+struct BlockRef {
+  int page, lo, hi, base;
+};
+
+__device__ inline BlockRef block_ref(const SeqInfo& si, const int32_t* hist_row,
+                                     const int32_t* live_row, int b) {
+  BlockRef r;
+  if (b < si.n_hist_pages) {
+    r.page = hist_row[b];
+    r.lo = 0;
+    r.hi = min(PS, si.n_hist - b * PS);
+    r.base = b * PS;
+  } else {
+    int lb = b - si.n_hist_pages;
+    int s0 = lb * PS;
+    r.page = live_row[lb];
+    r.lo = max(0, si.live_head - s0);
+    r.hi = min(PS, si.live_head + si.n_live - s0);
+    r.base = si.n_hist + s0 - si.live_head;
+  }
+  return r;
+}
+
+__device__ inline void set_error(const Dev& d, int bits) { atomicOr(&d.g->err, bits); }
+
+// ---------------------------------------------------------------------------
+// PTX helpers: mbarrier and bulk (TMA) copies global -> shared.
+// ---------------------------------------------------------------------------
+__device__ inline uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ inline void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+
+__device__ inline void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ inline void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ inline void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ inline void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ inline bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: returns false (and records KVC_DERR_WAIT) if the phase does
+// not complete within WAIT_LIMIT_CYCLES.
+__device__ inline bool mbar_wait(const Dev& d, uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > WAIT_LIMIT_CYCLES) {
+      set_error(d, KVC_DERR_WAIT);
+      return false;
+    }
+  }
+  return true;
+}
+
+// 1-D bulk copy (TMA engine): `bytes` (multiple of 16) from 16-byte aligned
+// global memory into 16-byte aligned shared memory, completing on `bar`.
+__device__ inline void bulk_g2s(void* dst_smem, const void* src_gmem, uint32_t bytes,
+                                uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(smem_u32(dst_smem)),
+      "l"(src_gmem), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Small numeric helpers.
+// ---------------------------------------------------------------------------
+__device__ inline float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ inline float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+template <typename T>
+__device__ inline T from_float(float x);
+template <>
+__device__ inline float from_float<float>(float x) {
+  return x;
+}
+template <>
+__device__ inline __nv_bfloat16 from_float<__nv_bfloat16>(float x) {
+  return __float2bfloat16_rn(x);
+}
+
+template <typename T>
+__device__ inline float to_float(T x);
+template <>
+__device__ inline float to_float<float>(float x) {
+  return x;
+}
+template <>
+__device__ inline float to_float<__nv_bfloat16>(__nv_bfloat16 x) {
+  return __bfloat162float(x);
+}
+
+// exp2 with -inf - -inf treated as 0 weight.
+__device__ inline float exp2_safe(float x, float m) {
+  return (m == -INFINITY) ? 0.f : exp2f(x - m);
+}
+
+// ---------------------------------------------------------------------------
+// Launchers (defined in the .cu files).
+// ---------------------------------------------------------------------------
+struct AppendArgs {
+  int32_t n_seq;
+  int32_t total;
+  int32_t dec_target, pf_target;   // desired split-K item counts
+  int32_t dec_min_blocks, pf_min_blocks;
+  int32_t sessions[MAX_SEQ];
+  int32_t cu[MAX_SEQ + 1];
+};
+
+struct SeqArgs {
+  int32_t n_seq;
+  int32_t sessions[MAX_SEQ];
+};
+
+cudaError_t launch_init(const Dev& d, double rope_base, cudaStream_t s);
+cudaError_t launch_append(const Dev& d, const AppendArgs& a, const uint8_t* types, const void* k,
+                          const void* v, cudaStream_t s);
+cudaError_t launch_evict(const Dev& d, const SeqArgs& a, int64_t* resident_out, cudaStream_t s);
+cudaError_t launch_release(const Dev& d, const SeqArgs& a, cudaStream_t s);
+cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
+                               cudaStream_t s);
+cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
+                                int max_t, cudaStream_t s);
+int decode_grid_ctas(const Dev& d);
+int prefill_grid_ctas(const Dev& d);
+
+}  // namespace kvc

@@ -1,0 +1,226 @@
+"""GPU parity: the CUDA path against the oracle on the same seeded inputs.
+
+Bit-exact: eviction masks (retained position lists), resident counts, page
+tables, live head/size and per-slot {position, type, unit}.  Floating point:
+|gpu - ref| <= atol + rtol |ref| elementwise (bf16: 2e-2 + 1e-2 |ref|; fp32:
+1e-4 + 1e-4 |ref|) and a normwise bound (bf16 1e-2, fp32 1e-5); the reference is
+the float64 oracle on the same rounded inputs.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from harness import Lockstep, assert_close, compare_state  # noqa: E402
+from synth import script as S  # noqa: E402
+from synth import values as V  # noqa: E402
+from synth.driver import Driver, cache_sizing  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2609_31224_gb300 import build
+    from synth import gpu
+    build.build()
+    gpu.build()
+
+
+def test_device_generator_matches_numpy():
+    from synth import gpu
+    for dtype in ("bf16", "f32"):
+        sess = torch.tensor([0, 3, 3, 7], dtype=torch.int32, device="cuda")
+        pos = torch.tensor([0, 5, 4095, 123456], dtype=torch.int32, device="cuda")
+        t = torch.empty((3, 4, 8, 128), dtype=torch.bfloat16 if dtype == "bf16" else torch.float32,
+                        device="cuda")
+        for tag, scale in ((V.TAG_K, 1.0), (V.TAG_Q, 0.25)):
+            gpu.fill(t, dtype, 11, tag, sess, pos, scale)
+            got = t.float().cpu().numpy()
+            want = V.values(11, tag, sess.cpu().numpy()[None, :, None, None],
+                            np.arange(3)[:, None, None, None],
+                            pos.cpu().numpy()[None, :, None, None],
+                            np.arange(8)[None, None, :, None], np.arange(128)[None, None, None, :],
+                            dtype, scale)
+            assert np.array_equal(got, want)
+
+
+def _lockstep(w, n_units=None, sizing=None):
+    scripts = S.workload_scripts(w)
+    if n_units is not None:
+        for sc in scripts:
+            sc.n_transcript = sc.n_transcript[:n_units]
+            sc.n_text = sc.n_text[:n_units]
+    drv = Driver(w, scripts, sizing=sizing)
+    return Lockstep(drv, w), scripts
+
+
+def test_tiny_f32_every_call_every_evict():
+    """60 units, fp32: every attention output and every post-evict state."""
+    ls, scripts = _lockstep(S.TINY_F32)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda *a: True)
+    assert ls.n_compared > 60 * 6
+    st = ls.drv.cache.export_state(0)
+    assert st["resident"] <= 512 and st["n_evicted"] > 0
+
+
+def test_tiny_f32_prefix_window0_floor_budget():
+    w = S.TINY_F32.with_(prefix_len=37, window=0, budget=0, seed=3)
+    ls, _ = _lockstep(w, n_units=25)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda *a: True)
+    st = ls.drv.cache.export_state(0)
+    # floor budget: only prefix + transcripts remain
+    assert all(t in (2, 3) or u < 0 for t, u in zip(st["type"], st["unit"]))
+
+
+@pytest.mark.parametrize("budget,window,seed", [(64, 1, 1), (200, 3, 2), (-1, 5, 4),
+                                                (17, 0, 5), (1000, 50, 6)])
+def test_small_bf16_mixed_segments(budget, window, seed):
+    """bf16, 2 layers, 3 sessions with offsets, empty/long segments and speaking turns."""
+    w = S.SINGLE_BF16.with_(layers=2, n_sessions=3, offset_max=4, budget=budget,
+                            window=window, seed=seed, p_no_segment=0.1, p_long_segment=0.1,
+                            turn_period=12, turn_jitter=2, prefix_len=5)
+    ls, _ = _lockstep(w, n_units=40)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda step, kind, i, layer: layer == 1 or step % 5 == 0)
+    assert ls.n_compared > 100
+
+
+def test_sharp_attention_bf16():
+    """Larger query scale makes the softmax peaked, so a wrong key order shows."""
+    w = S.SINGLE_BF16.with_(layers=1, n_sessions=2, budget=96, window=2, seed=9, q_scale=6.0,
+                            turn_period=10, turn_jitter=1)
+    ls, _ = _lockstep(w, n_units=30)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda *a: True)
+    assert max(s["max_abs"] for s in ls.stats) > 0  # outputs were compared
+
+
+def test_single_session_full_size_metadata_and_sampled_attention():
+    """600 units, 32 layers, B=4096, W=10: every evict bit-exact; attention sampled."""
+    ls, _ = _lockstep(S.SINGLE_BF16)
+    samples = {0, 1, 50, 186, 187, 300, 420, 599}
+    for step in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda st, kind, i, layer: st in samples and
+                    (layer in (0, 31) or (kind == "decode" and i == 1 and layer == 17)))
+    st = ls.drv.cache.export_state(0)
+    assert st["resident"] <= 4096
+    assert st["peak_resident"] > 4096
+
+
+def test_batch64_sampled_at_full_size():
+    """64 sessions, offsets U{0..300}: state of every session bit-exact at sampled steps;
+    attention of sampled sessions/layers in the launch configuration of the benchmark."""
+    w = S.BATCH64_BF16
+    scripts = S.workload_scripts(w)
+    drv = Driver(w, scripts)
+    ls = Lockstep(drv, w)
+    stop = S.steady_state_step(w, scripts) + 3
+    check = set(range(0, stop, 97)) | {stop - 1}
+    for step in range(stop):
+        if step in check or step >= stop - 3:
+            ls.run_step(attn_pred=lambda st, kind, i, layer: st >= stop - 2 and
+                        layer in (0, 13, 31) and i in (0, 1, 4),
+                        session_pred=lambda s: s % 21 == 0)
+        else:
+            # Oracle replays the policy without comparing every state.
+            ls.run_step(attn_pred=None, check_state=False)
+    assert ls.n_compared >= 12
+
+
+def test_compaction_is_a_pure_move():
+    """Stored K/V of retained positions are byte-identical before and after evict."""
+    w = S.SINGLE_BF16.with_(layers=2, n_sessions=2, budget=100, window=2, seed=12)
+    scripts = S.workload_scripts(w)
+    for sc in scripts:
+        sc.n_transcript = sc.n_transcript[:20]
+        sc.n_text = sc.n_text[:20]
+    drv = Driver(w, scripts)
+    moved = 0
+    for _ in range(len(drv.sched)):
+        st = drv.prepare_step()
+        for c in st.calls:
+            drv.run_call(c)
+        before = {}
+        for s in st.evict_sessions.tolist():
+            meta = drv.cache.export_state(s)
+            for layer in (0, 1):
+                k, v = drv.cache.export_kv(s, layer)
+                before[(s, layer)] = dict(zip(meta["pos"], zip(k, v)))
+        drv.cache.evict(st.evict_sessions)
+        for s in st.evict_sessions.tolist():
+            meta = drv.cache.export_state(s)
+            for layer in (0, 1):
+                k, v = drv.cache.export_kv(s, layer)
+                for p, kk, vv in zip(meta["pos"], k, v):
+                    kb, vb = before[(s, layer)][p]
+                    assert np.array_equal(kk, kb) and np.array_equal(vv, vb)
+                    moved += 1
+    assert moved > 0
+
+
+def test_stored_keys_match_oracle_rotation():
+    """K is stored rotated at its original position (within one storage ulp)."""
+    from oracle.numerics import round_bf16
+    from oracle.rope import rope
+    w = S.SINGLE_BF16.with_(layers=1, n_sessions=1, budget=-1, seed=2)
+    scripts = S.workload_scripts(w)
+    for sc in scripts:
+        sc.n_transcript = sc.n_transcript[:8]
+        sc.n_text = sc.n_text[:8]
+    drv = Driver(w, scripts)
+    for _ in range(len(drv.sched)):
+        drv.run_step(drv.prepare_step(), attention=False)
+    meta = drv.cache.export_state(0)
+    k, v = drv.cache.export_kv(0, 0)
+    pos = np.asarray(meta["pos"])
+    raw = V.layer_tensor(w.seed, V.TAG_K, 0, 0, pos, w.kv_heads, w.head_dim, "bf16")
+    want = round_bf16(rope(raw, pos[:, None], w.rope_base))
+    ulp = np.abs(want) * 2.0 ** -7 + 1e-30
+    assert (np.abs(k - want) <= ulp).all()
+    assert np.mean(k == want) > 0.99
+    assert np.array_equal(v, V.layer_tensor(w.seed, V.TAG_V, 0, 0, pos, w.kv_heads,
+                                            w.head_dim, "bf16"))
+
+
+def test_error_codes():
+    from paper_2609_31224_gb300 import KVCache, KvcError
+    c = KVCache(n_sessions=2, layers=1, q_heads=4, kv_heads=1, head_dim=64, budget=8, window=0,
+                dtype="f32", n_pages=3, max_pages_per_session=4, max_positions=100,
+                max_seq_per_call=2, max_tokens_per_call=64)
+    q = torch.zeros((64, 4, 64), device="cuda")
+    out = torch.zeros_like(q)
+    with pytest.raises(KvcError) as e:
+        c.attn_decode(0, q, out)
+    assert e.value.code == -4  # no append yet
+    types = torch.zeros(64, dtype=torch.uint8, device="cuda")
+    kv = torch.zeros((1, 64, 1, 64), device="cuda")
+    with pytest.raises(KvcError) as e:
+        c.append_chunk([0], [0, 60], types, kv, kv)
+    assert e.value.code == -2  # 60 tokens need 4 pages, the pool has 3
+    c.append_chunk([0], [0, 20], types, kv, kv)
+    with pytest.raises(KvcError) as e:
+        c.attn_decode(0, q, out)
+    assert e.value.code == -4  # decode needs one token per session
+    with pytest.raises(KvcError) as e:
+        c.append_chunk([1], [0, 20], types, kv, kv)
+    assert e.value.code == -2  # pool has 3 pages, 2 in use
+    with pytest.raises(KvcError) as e:
+        c.append_chunk([0, 0], [0, 1, 2], types, kv, kv)
+    assert e.value.code == -1  # repeated session
+    with pytest.raises(KvcError) as e:
+        c.attn_prefill_chunk(5, q, out)
+    assert e.value.code == -1  # bad layer
+    c.evict([0])
+    with pytest.raises(KvcError) as e:
+        c.attn_prefill_chunk(0, q, out)
+    assert e.value.code == -4  # evict invalidates the queries
+    free, err = c.device_status()
+    assert err == 0 and free >= 1
+    c.release([0])
+    free, err = c.device_status()
+    assert free == 3
