@@ -1,0 +1,438 @@
+"""Benchmark: audio-seconds processed per second through the whole hot path
+(append + chunked-prefill and decode attention of every layer + eviction), on
+the 64-session ten-minute workload (32 layers, 32/8 heads, head_dim 128, bf16,
+B=4096, W=10, session starts U{0..300} s).
+
+One step advances every active session by one one-second unit.  The cache is
+first brought (untimed, append + evict only: attention changes no state) to
+the step where every session is active and at its budget; W warm-up steps
+follow, then K timed steps.  Per-step K/V traffic is hundreds of GB, far
+above the 129 MB L2, so no flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  N > 1 (torchrun): every rank runs an
+independent replica of the workload (sessions are independent; no
+collective on the data path): weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "audio-seconds processed/sec (evict+attn, all layers); HBM GB/s vs GB300 peak"
+UNIT = "audio-s/s"
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# -- clocks sampled during the timed region ------------------------------------------------
+class Clocks:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# -- algorithmic bytes -------------------------------------------------------------------------
+def step_bytes(w, drv, st, prev_resident: dict) -> tuple[float, float, int]:
+    """(attention+append bytes of the step, bytes of its first full-batch decode round per
+    layer launch, number of decode sessions in that round)."""
+    esz = 2 if w.dtype == "bf16" else 4
+    per_pos_layer = w.kv_heads * w.head_dim * 2 * esz           # K+V of one position, one layer
+    q_row = w.q_heads * w.head_dim * esz
+    total = 0.0
+    n_now = {s: prev_resident.get(s, 0) for s, _ in st.pairs}
+    round0_bytes, round0_n = 0.0, 0
+    dec_round = 0
+    for c in st.calls:
+        cnt = np.diff(c.cu)
+        for s, t in zip(c.sessions.tolist(), cnt.tolist()):
+            n_now[s] += t
+        total += int(c.cu[-1]) * w.layers * per_pos_layer        # append: K+V written
+        if c.kind == "prefix":
+            continue
+        keys = sum(n_now[s] for s in c.sessions.tolist())
+        per_launch = keys * per_pos_layer + 2 * int(c.cu[-1]) * q_row
+        total += w.layers * per_launch
+        if c.kind == "decode":
+            if dec_round == 0:
+                round0_bytes, round0_n = per_launch, len(c.sessions)
+            dec_round += 1
+    return total, round0_bytes, round0_n
+
+
+def run_ours(args, rank: int, world: int, local_rank: int):
+    import torch
+    from synth import script as S
+    from synth.driver import Driver
+
+    torch.cuda.set_device(local_rank)
+    w = S.BATCH64_BF16
+    scripts = S.workload_scripts(w)
+    drv = Driver(w, scripts)
+    start = args.start if args.start is not None else S.steady_state_step(w, scripts)
+    n_steps_total = len(drv.sched)
+    assert start - args.warmup >= 0 and start + args.steps <= n_steps_total
+    e2e_steps = args.e2e_steps if args.e2e_steps is not None else min(args.steps, 8)
+    assert start + args.steps + e2e_steps <= n_steps_total
+
+    # 1. Bring the cache to the step before the warm-up (append + evict only).
+    drv.fast_forward(start - args.warmup)
+    torch.cuda.synchronize()
+
+    # 2. Inputs of the warm-up and timed steps, resident on the device.
+    warm = [drv.prepare_step() for _ in range(args.warmup)]
+    timed = [drv.prepare_step() for _ in range(args.steps)]
+    n_res_buf = torch.zeros((args.steps + 1, w.n_sessions), dtype=torch.int64, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    idx_of = {id(st): torch.as_tensor(st.evict_sessions.astype(np.int64), device="cuda")
+              for st in warm + timed}
+
+    def snapshot_resident(row, st):
+        idx = idx_of[id(st)]
+        n_res_buf[row].index_copy_(0, idx, drv.resident_out[:len(idx)])
+
+    for st in warm:
+        drv.run_step(st)
+    snapshot_resident(0, warm[-1])
+    torch.cuda.synchronize()
+
+    # 3. Timed steps.  Events around the first full-batch decode round (all layers) of every
+    #    step give the decode kernel's live per-launch duration.
+    dec_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in timed]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches = 0
+    clocks = Clocks(local_rank)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    torch.cuda.nvtx.range_push("timed")
+    t0.record(stream)
+    for i, st in enumerate(timed):
+        first_dec = next((c for c in st.calls if c.kind == "decode"), None)
+        for c in st.calls:
+            if c is first_dec:
+                drv.cache.append_chunk(c.sessions, c.cu, c.types, c.k, c.v)
+                dec_ev[i][0].record(stream)
+                for layer in range(w.layers):
+                    drv.cache.attn_decode(layer, c.q[layer], c.out)
+                dec_ev[i][1].record(stream)
+                launches += 2 + w.layers
+            else:
+                launches += drv.run_call(c)
+        drv.cache.evict(st.evict_sessions, drv.resident_out)
+        launches += 2
+        snapshot_resident(i + 1, st)
+    t1.record(stream)
+    torch.cuda.nvtx.range_pop()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    elapsed_ms = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([elapsed_ms], dtype=torch.float64, device="cuda")
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        elapsed_ms = float(tt.item())
+    audio_s = sum(len(st.pairs) for st in timed)          # one unit = one audio second
+    value_rank = audio_s / (elapsed_ms / 1e3)
+
+    # Algorithmic bytes (attention reads every resident K/V byte once per call per layer).
+    res = n_res_buf.cpu().numpy()
+    tot_bytes, dec_bytes, dec_times = 0.0, [], []
+    for i, st in enumerate(timed):
+        prev = {s: int(res[i, s]) for s, _ in st.pairs}
+        b, rb, _ = step_bytes(w, drv, st, prev)
+        tot_bytes += b
+        if rb:
+            dec_bytes.append(rb)
+            dec_times.append(dec_ev[i][0].elapsed_time(dec_ev[i][1]) / w.layers)
+    del timed, warm
+    torch.cuda.empty_cache()
+
+    # 4. End to end through the public API: inputs copied from pinned host memory every
+    #    step, the step's result (resident counts and last-layer outputs) read back.
+    e2e = run_e2e(drv, w, e2e_steps, world)
+
+    peak, peak_kind = load_peaks()
+    dec_gbs = (sum(dec_bytes) / 1e9) / (sum(dec_times) / 1e3) if dec_times else None
+    out = {
+        "metric": METRIC,
+        "value": value_rank * world,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": elapsed_ms / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": w.dtype,
+        "data": "synthetic (seeded SplitMix64 Irwin-Hall values, PCG64 session scripts)",
+        "config": {
+            "workload": w.name,
+            "sessions": w.n_sessions, "layers": w.layers, "q_heads": w.q_heads,
+            "kv_heads": w.kv_heads, "head_dim": w.head_dim, "page_size": w.page_size,
+            "budget": w.budget, "window": w.window, "units_per_session": w.units,
+            "offsets": f"U{{0..{w.offset_max}}}", "timed_steps": [start, start + args.steps],
+            "audio_seconds_timed_per_gpu": audio_s,
+            "l2": "no flush: per-step K/V traffic >> 129 MB L2",
+            "parallelism": f"replicas x{world}",
+        },
+        "path_hbm_gbs": (tot_bytes / 1e9) / (elapsed_ms / 1e3),
+        "path_frac_of_peak": (tot_bytes / 1e9) / (elapsed_ms / 1e3) / peak,
+        "roofline": {
+            "kernel": "attn_decode_kernel",
+            "bound": "hbm",
+            "achieved": dec_gbs,
+            "peak": peak,
+            "peak_kind": f"{peak_kind} copy bandwidth",
+            "unit": "GB/s",
+            "frac": (dec_gbs / peak) if dec_gbs else None,
+            "traffic": None,
+            "algorithmic_bytes_per_launch": (sum(dec_bytes) / len(dec_bytes)) if dec_bytes else None,
+            "avg_launch_us": (1e3 * sum(dec_times) / len(dec_times)) if dec_times else None,
+        },
+        "e2e": e2e,
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    return out
+
+
+def run_e2e(drv, w, n_steps: int, world: int) -> dict:
+    import torch
+    stream = torch.cuda.current_stream()
+    steps = [drv.prepare_step() for _ in range(n_steps)]
+    # Move every input to pinned host memory; keep same-shaped device buffers.
+    host, dev = [], []
+    for st in steps:
+        hs, ds = [], []
+        for c in st.calls:
+            names = ["types", "k", "v"] + (["q"] if c.q is not None else [])
+            h = {n: getattr(c, n).cpu().pin_memory() for n in names}
+            hs.append(h)
+            ds.append({n: getattr(c, n) for n in names})
+        host.append(hs)
+        dev.append(ds)
+    res_host = torch.empty(w.n_sessions, dtype=torch.int64).pin_memory()
+    out_host = [[torch.empty(c.out.shape, dtype=c.out.dtype).pin_memory() if c.out is not None
+                 else None for c in st.calls] for st in steps]
+    h2d = sum(t.numel() * t.element_size() for hs in host[0] for t in hs.values())
+    d2h = res_host.numel() * 8 + sum(o.numel() * o.element_size()
+                                     for o in out_host[0] if o is not None)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t0 = time.perf_counter()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    h2d_total, d2h_total = 0, 0
+    for si, st in enumerate(steps):
+        for ci, c in enumerate(st.calls):
+            for n, t in host[si][ci].items():
+                dev[si][ci][n].copy_(t, non_blocking=True)
+                h2d_total += t.numel() * t.element_size()
+            drv.run_call(c)
+            if c.out is not None:
+                out_host[si][ci].copy_(c.out, non_blocking=True)
+                d2h_total += c.out.numel() * c.out.element_size()
+        drv.cache.evict(st.evict_sessions, drv.resident_out)
+        n = len(st.evict_sessions)
+        res_host[:n].copy_(drv.resident_out[:n], non_blocking=True)
+        d2h_total += n * 8
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    wall = time.perf_counter() - t0
+    if world > 1:
+        tt = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = float(tt.item())
+    audio_s = sum(len(st.pairs) for st in steps)
+    return {"value": world * audio_s / (ms / 1e3), "unit": UNIT,
+            "h2d_bytes_per_step": h2d_total / n_steps, "d2h_bytes_per_step": d2h_total / n_steps,
+            "steps": n_steps, "host_wall_s": wall}
+
+
+# -- the oracle on the host cores -----------------------------------------------------------------
+def oracle_sample(layers_sampled: int = 1, session: int = 0, start: int | None = None) -> dict:
+    """Time the CPU oracle on one session's unit at the benchmark's steady state, for
+    `layers_sampled` of its 32 layers (policy + every attention call of those layers);
+    scaled to audio-s/s by the sampled fraction of one unit."""
+    from oracle.cache import OracleCache, OracleConfig
+    from synth import script as S
+    from synth import values as V
+
+    w = S.BATCH64_BF16
+    scripts = S.workload_scripts(w)
+    sc = scripts[session]
+    start = S.steady_state_step(w, scripts) if start is None else start
+    unit = start - sc.offset
+    orc = OracleCache(OracleConfig(n_sessions=1, layers=w.layers, q_heads=w.q_heads,
+                                   kv_heads=w.kv_heads, head_dim=w.head_dim,
+                                   page_size=w.page_size, budget=w.budget, window=w.window,
+                                   dtype=w.dtype, rope_base=w.rope_base, n_pages=1 << 20))
+    for u in range(unit):           # state before the sampled unit (untimed)
+        orc.append_chunk([0], [sc.unit_types(u)])
+        orc.evict([0])
+
+    def kv(s, layer, pos):
+        return (V.layer_tensor(w.seed, V.TAG_K, session, layer, pos, w.kv_heads, w.head_dim,
+                               w.dtype), V.layer_tensor(w.seed, V.TAG_V, session, layer, pos,
+                                                        w.kv_heads, w.head_dim, w.dtype))
+
+    t0 = time.perf_counter()
+    chunks = [sc.prefill_types()] + [sc.decode_types(unit)[i:i + 1]
+                                     for i in range(len(sc.decode_types(unit)))]
+    for types in chunks:
+        orc.append_chunk([0], [types])
+        pos = orc.last_append[0][1]
+        for layer in range(layers_sampled):
+            q = V.layer_tensor(w.seed, V.TAG_Q, session, layer, pos, w.q_heads, w.head_dim,
+                               w.dtype)
+            orc.attend(layer, [q], kv)
+    orc.evict([0])
+    dt = time.perf_counter() - t0
+    frac = layers_sampled / w.layers
+    try:
+        from threadpoolctl import threadpool_info
+        cores = max([i.get("num_threads", 1) for i in threadpool_info()] + [1])
+    except Exception:
+        cores = len(os.sched_getaffinity(0))
+    return {"value": frac / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "seconds": dt,
+            "sample": f"session {session}, unit {unit} (step {start}) of {w.name}: eviction rule "
+                      f"+ {len(chunks)} attention calls x {layers_sampled}/{w.layers} layers "
+                      f"in float64; value = sampled fraction of one audio-second / time"}
+
+
+def run_reference(args, rank: int, world: int):
+    """The oracle timed as the reference arm (host cores), same metric and unit."""
+    if rank != 0:
+        return None
+    samples = [oracle_sample(layers_sampled=1, session=(i % 64)) for i in range(args.steps)]
+    for _ in range(0):
+        pass
+    total_audio = sum(s["value"] * s["seconds"] for s in samples)
+    total_t = sum(s["seconds"] for s in samples)
+    v = total_audio / total_t
+    return {
+        "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * total_t / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "impl": "reference",
+        "config": {"workload": "batch64-bf16-32L-32q8kv-d128-600u-off300-B4096-W10",
+                   "sample": "1 of 32 layers of one session-unit per step"},
+        "cpu_baseline": {"value": v, "unit": UNIT, "kind": "oracle",
+                         "cores": samples[0]["cores"], "sample": samples[0]["sample"]},
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--start", type=int, default=None, help="first timed step of the schedule")
+    ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local_rank = int(os.environ.get("LOCAL_RANK", 0))
+    if world > 1 and args.impl == "ours":
+        import torch
+        torch.distributed.init_process_group(
+            backend="nccl" if torch.cuda.is_available() else "gloo")
+
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+        if out is not None:
+            print(json.dumps(out))
+        return
+
+    from __graft_entry__ import build
+    build()
+    out = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            out["cpu_baseline"] = oracle_sample(layers_sampled=2)
+        print(json.dumps(out))
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -320,7 +320,7 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, const i
   a.total = total;
   a.dec_target = ctx->dec_target;
   a.pf_target = ctx->pf_target;
-  a.dec_min_blocks = 4;
+  a.dec_min_blocks = 8;
   a.pf_min_blocks = 4;
   for (int i = 0; i < n_seq; ++i) a.sessions[i] = h_sessions[i];
   for (int i = 0; i <= n_seq; ++i) a.cu[i] = h_cu_tokens[i];

@@ -19,6 +19,7 @@ constexpr unsigned FULL = 0xFFFFFFFFu;
 constexpr int DEC_WARPS = 4;
 constexpr int DEC_THREADS = DEC_WARPS * 32;
 constexpr int G = 4;  // query heads per KV head
+static_assert(DEC_WARPS == G, "the split-K merge maps one warp to one query row");
 constexpr float LOG2E = 1.4426950408889634f;
 
 template <typename T, int D, int STAGES>
@@ -31,8 +32,12 @@ struct DecCfg {
   static constexpr int TILE = PS * ROW_BYTES;  // one page of one head: 4 KiB
   // shared memory per warp: STAGES x (K tile + V tile) + scores + probs + alpha
   static constexpr int WARP_BYTES = STAGES * 2 * TILE + (G * PS + PS * G + G) * 4 + 16;
+  // The cross-warp merge reuses the stage buffers once every warp is done.
   static constexpr int MERGE_BYTES = DEC_WARPS * G * (D + 2) * 4;
-  static constexpr int SMEM = DEC_WARPS * WARP_BYTES + MERGE_BYTES + DEC_WARPS * STAGES * 8 + 64;
+  static_assert(MERGE_BYTES <= DEC_WARPS * WARP_BYTES, "merge area must fit in the stages");
+  static constexpr int MAX_CHUNKS = 64;  // split-K chunks per session (work-list cap)
+  static constexpr int SMEM = DEC_WARPS * WARP_BYTES + DEC_WARPS * STAGES * 8 +
+                              MAX_CHUNKS * G * 4 + 64;
 };
 
 template <typename T>
@@ -75,11 +80,11 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
   float* s_sc = reinterpret_cast<float*>(wbase + STAGES * 2 * C::TILE);  // [G][PS]
   float* s_p = s_sc + G * PS;                                        // [PS][G]
   float* s_alpha = s_p + PS * G;                                     // [G]
-  float* m_o = reinterpret_cast<float*>(smem + DEC_WARPS * C::WARP_BYTES);  // [W][G][D]
-  float* m_ml = m_o + DEC_WARPS * G * D;                                     // [W][G][2]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + DEC_WARPS * C::WARP_BYTES +
-                                               C::MERGE_BYTES);
+  float* m_o = reinterpret_cast<float*>(smem);   // [W][G][D], aliases the stages
+  float* m_ml = m_o + DEC_WARPS * G * D;          // [W][G][2]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + DEC_WARPS * C::WARP_BYTES);
   uint64_t* wbars = bars + warp * STAGES;
+  float* s_scale = reinterpret_cast<float*>(bars + DEC_WARPS * STAGES);  // [MAX_CHUNKS][G]
   __shared__ int s_last, s_abort;
 
   if (lane == 0) {
@@ -138,6 +143,7 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
       bulk_g2s(dst + C::TILE, kp + d.kv_heads * head_stride, C::TILE, &wbars[st]);
     };
     if (lane == 0) {
+      fence_proxy_async_smem();  // the stage buffers were written by the previous merge
       for (int k = 0; k < min(STAGES, n_my); ++k) issue(k);
     }
 
@@ -257,7 +263,8 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
     }
     loads += n_my;
 
-    // Merge the four warps' partial softmax states.
+    // Merge the four warps' partial softmax states (stage buffers are free now).
+    __syncthreads();
     if ((lane & 7) == 0) {
       m_ml[(warp * G + (lane >> 3)) * 2 + 0] = m_run;
       m_ml[(warp * G + (lane >> 3)) * 2 + 1] = l_run;
@@ -301,21 +308,50 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
       __syncthreads();
       if (s_last) {
         __threadfence();
+        // Log-sum-exp merge of the session's chunks: warp g reduces row g's maxima and
+        // sums over the chunks (lanes stride the chunks), leaving each chunk's weight
+        // divided by the total in shared memory; then all threads sum the weighted
+        // partial outputs over (row, dim) with independent loads in flight.
         const int s0 = si.dec_base * d.kv_heads + head;
+        const int nch = si.dec_chunks;
+        {
+          const int g = warp;  // DEC_WARPS == G
+          float M = -INFINITY;
+          for (int ch = lane; ch < nch; ch += 32)
+            M = fmaxf(M, __ldcg(&d.dec_part_ml[(size_t)(s0 + ch * d.kv_heads) * G + g]).x);
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(FULL, M, o));
+          float L = 0.f;
+          for (int ch = lane; ch < nch; ch += 32) {
+            const float2 ml = __ldcg(&d.dec_part_ml[(size_t)(s0 + ch * d.kv_heads) * G + g]);
+            const float sc = exp2_safe(ml.x, M);
+            s_scale[ch * G + g] = sc;
+            L += ml.y * sc;
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(FULL, L, o);
+          const float inv = 1.f / L;
+          __syncwarp();
+          for (int ch = lane; ch < nch; ch += 32) s_scale[ch * G + g] *= inv;
+        }
+        __syncthreads();
         for (int e = tid; e < G * D; e += DEC_THREADS) {
           const int g = e / D, dd = e % D;
-          float M = -INFINITY;
-          for (int ch = 0; ch < si.dec_chunks; ++ch)
-            M = fmaxf(M, __ldcg(&d.dec_part_ml[(size_t)(s0 + ch * d.kv_heads) * G + g]).x);
-          float L = 0.f, O = 0.f;
-          for (int ch = 0; ch < si.dec_chunks; ++ch) {
-            const size_t sl = (size_t)(s0 + ch * d.kv_heads);
-            const float2 ml = __ldcg(&d.dec_part_ml[sl * G + g]);
-            const float sc = exp2_safe(ml.x, M);
-            L += ml.y * sc;
-            O += __ldcg(&d.dec_part_o[(sl * G + g) * D + dd]) * sc;
+          float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
+          int ch = 0;
+          for (; ch + 4 <= nch; ch += 4) {
+            const size_t b0 = ((size_t)(s0 + ch * d.kv_heads) * G + g) * D + dd;
+            const size_t st = (size_t)d.kv_heads * G * D;
+            O0 += __ldcg(&d.dec_part_o[b0]) * s_scale[ch * G + g];
+            O1 += __ldcg(&d.dec_part_o[b0 + st]) * s_scale[(ch + 1) * G + g];
+            O2 += __ldcg(&d.dec_part_o[b0 + 2 * st]) * s_scale[(ch + 2) * G + g];
+            O3 += __ldcg(&d.dec_part_o[b0 + 3 * st]) * s_scale[(ch + 3) * G + g];
           }
-          out[((size_t)si.q_row0 * d.q_heads + head * G + g) * D + dd] = from_float<T>(O / L);
+          for (; ch < nch; ++ch)
+            O0 += __ldcg(&d.dec_part_o[((size_t)(s0 + ch * d.kv_heads) * G + g) * D + dd]) *
+                  s_scale[ch * G + g];
+          out[((size_t)si.q_row0 * d.q_heads + head * G + g) * D + dd] =
+              from_float<T>((O0 + O1) + (O2 + O3));
         }
         if (tid == 0) d.dec_count[itm.seq * d.kv_heads + head] = 0;
       }

@@ -111,6 +111,7 @@ struct Dev {
 };
 
 constexpr int PF_MAX_TOKENS = 32;  // tokens per session per prefill call
+constexpr int MAX_CHUNKS_PER_SEQ = 64;  // split-K chunks per session and call
 
 __host__ __device__ inline size_t pool_offset_elems(const Dev& d, int page, int layer, int kv,
                                                     int head, int slot) {

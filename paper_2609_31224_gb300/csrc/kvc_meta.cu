@@ -173,7 +173,7 @@ __device__ void build_worklist(const Dev& d, int n_seq, int nb, int target, int 
   int per = max(min_blocks, (int)(((int64_t)total_blocks * d.kv_heads + target - 1) / target));
   int chunks = 0, base = 0, total_items = 0;
   for (int iter = 0; iter < 32; ++iter) {
-    chunks = (i < n_seq) ? (nb + per - 1) / per : 0;
+    chunks = (i < n_seq) ? min(MAX_CHUNKS_PER_SEQ, (nb + per - 1) / per) : 0;
     base = block_exclusive_scan(chunks, &total_items, s_warp);
     if ((int64_t)total_items * d.kv_heads <= max_items) break;
     per *= 2;

@@ -61,6 +61,7 @@ class Call:
     cu: np.ndarray                 # int32 token offsets
     positions: list                # per session, positions of its tokens
     types: object = None           # device uint8 [total]
+    types_host: np.ndarray = None  # the same, on the host
     k: object = None               # device [L][total][Hkv][D]
     v: object = None
     q: object = None               # device [L][total][Hq][D]
@@ -121,8 +122,8 @@ class Driver:
             tok_sess += [s] * n
             tok_pos += p
         c = Call(kind=kind, sessions=sess, cu=cu, positions=positions)
-        c.types = torch.as_tensor(np.concatenate(types_per_session).astype(np.uint8),
-                                  device=self.device)
+        c.types_host = np.concatenate(types_per_session).astype(np.uint8)
+        c.types = torch.as_tensor(c.types_host, device=self.device)
         c.k = self._fill(V.TAG_K, w.kv_heads, tok_sess, tok_pos, w.kv_scale)
         c.v = self._fill(V.TAG_V, w.kv_heads, tok_sess, tok_pos, w.kv_scale)
         if with_q:

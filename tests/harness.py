@@ -10,8 +10,9 @@ from synth import values as V
 TOL = {"bf16": (2e-2, 1e-2, 1e-2), "f32": (1e-4, 1e-4, 1e-5)}  # atol, rtol, normwise
 
 
-def assert_close(gpu: np.ndarray, ref: np.ndarray, dtype: str, what: str = "") -> dict:
-    atol, rtol, normwise = TOL[dtype]
+def assert_close(gpu: np.ndarray, ref: np.ndarray, dtype: str, what: str = "",
+                 tol=None) -> dict:
+    atol, rtol, normwise = TOL[dtype] if tol is None else tol
     gpu = np.asarray(gpu, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
     assert gpu.shape == ref.shape, (gpu.shape, ref.shape)
@@ -33,9 +34,10 @@ def compare_state(gpu_state: dict, ref_state: dict, what: str = "") -> None:
 
 
 class Lockstep:
-    def __init__(self, driver, w):
+    def __init__(self, driver, w, tol=None):
         self.drv = driver
         self.w = w
+        self.tol = tol
         self.orc = OracleCache(OracleConfig(
             n_sessions=w.n_sessions, layers=w.layers, q_heads=w.q_heads, kv_heads=w.kv_heads,
             head_dim=w.head_dim, page_size=w.page_size, budget=w.budget, window=w.window,
@@ -68,7 +70,7 @@ class Lockstep:
 
         def on_append(c):
             self.orc.append_chunk(c.sessions.tolist(),
-                                  [c.types.cpu().numpy()[c.cu[i]:c.cu[i + 1]]
+                                  [c.types_host[c.cu[i]:c.cu[i + 1]]
                                    for i in range(len(c.sessions))])
             call_idx[id(c)] = len(call_idx)
 
@@ -87,7 +89,8 @@ class Lockstep:
                 got = out[c.cu[i]:c.cu[i + 1]]
                 self.stats.append(assert_close(
                     got, ref, self.w.dtype,
-                    f"step {st.index} {c.kind} layer {layer} session {int(c.sessions[i])}"))
+                    f"step {st.index} {c.kind} layer {layer} session {int(c.sessions[i])}",
+                    self.tol))
                 self.n_compared += 1
 
         def on_evict(step):
