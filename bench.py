@@ -130,6 +130,11 @@ def run_ours(args, rank: int, world: int, local_rank: int):
 
     torch.cuda.set_device(local_rank)
     w = S.BATCH64_BF16
+    if args.sessions or args.layers:
+        # Reduced case of the same kernels (for profiler captures that must stay small).
+        w = w.with_(n_sessions=args.sessions or w.n_sessions, layers=args.layers or w.layers,
+                    name=f"{w.name}-reduced-{args.sessions or w.n_sessions}s-"
+                         f"{args.layers or w.layers}L")
     scripts = S.workload_scripts(w)
     drv = Driver(w, scripts)
     start = args.start if args.start is not None else S.steady_state_step(w, scripts)
@@ -404,6 +409,10 @@ def main():
     ap.add_argument("--start", type=int, default=None, help="first timed step of the schedule")
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sessions", type=int, default=None,
+                    help="reduced case for profiler captures (default: the full 64)")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="reduced case for profiler captures (default: the full 32)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
