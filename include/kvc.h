@@ -14,8 +14,9 @@
  *
  * Conventions for every call:
  *  - Device memory (pool, metadata workspace, q/k/v/out, types) is owned by
- *    the caller and must outlive the context.  The library never allocates
- *    device memory.
+ *    the caller and must outlive the context.  The library never calls a
+ *    device allocator; kvc_attn_decode_noalloc uses one fixed array that the
+ *    library itself defines.
  *  - Calls taking a stream are asynchronous on it (cudaStream_t passed as
  *    void*; NULL is the legacy default stream), except where a comment says
  *    "synchronises".
@@ -91,7 +92,7 @@ typedef struct kvc_config {
 } kvc_config;
 
 /* Supported shapes: (KVC_BF16, head_dim 128) and (KVC_F32, head_dim 64), with
- * G = Hq / Hkv in {1, 2, 4, 8} and page_size 16. */
+ * G = Hq / Hkv = 4 and page_size 16. */
 
 typedef struct kvc_session_info {
   int32_t pos_next;       /* next position id (= positions fed so far) */
@@ -169,6 +170,28 @@ int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out
  *   d_q     device [n_seq][Hq][D] un-rotated queries (call order of the append)
  *   d_out   device [n_seq][Hq][D] */
 int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void* stream);
+
+/* kvc_attn_decode without caller-provided scratch.  The paper has no
+ * counterpart.  It is for callers that cannot allocate device memory for
+ * scratch when they decode: for example a real-time duplex loop that must not
+ * stall on the implicit device synchronisation cudaMalloc and cudaFree can
+ * cause inside a one-second unit, or a host application whose device memory is
+ * owned by another framework that forbids allocations from outside it.
+ *
+ * Same arguments, layouts and result as kvc_attn_decode (within the attention
+ * tolerance: the split-K chunking differs).  The split-K partial results and
+ * arrival counters live in one fixed array in device global memory that the
+ * library defines (8.1 MiB; every GPU that loads the library holds it until the
+ * process exits), so this call allocates nothing.
+ *   - Limit: at most 4096 (session, kv-head) pairs per call, i.e. the last
+ *     append's n_seq * kv_heads <= 4096; larger calls return KVC_EINVAL with a
+ *     message and launch nothing.
+ *   - The first call on each device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - Every call shares the array and clears the counters it needs; calls whose
+ *     kernels can overlap on the GPU (other streams, other contexts in this
+ *     process) race on it, so serialise them. */
+int kvc_attn_decode_noalloc(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void* stream);
 
 /* Resident count of one session (n_hist + n_live), including the system
  * prefix and text (Sec. 3.3).  Synchronises the device. */

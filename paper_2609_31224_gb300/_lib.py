@@ -22,7 +22,8 @@ STATUS = {0: "KVC_OK", -1: "KVC_EINVAL", -2: "KVC_ENOMEM", -3: "KVC_ECUDA", -4: 
           -5: "KVC_EDEVICE"}
 
 EXPORTED = ["kvc_query_sizes", "kvc_create", "kvc_destroy", "kvc_append_chunk", "kvc_evict",
-            "kvc_attn_prefill_chunk", "kvc_attn_decode", "kvc_resident_size", "kvc_release",
+            "kvc_attn_prefill_chunk", "kvc_attn_decode", "kvc_attn_decode_noalloc",
+            "kvc_resident_size", "kvc_release",
             "kvc_export_state", "kvc_export_kv", "kvc_device_status", "kvc_last_error"]
 
 
@@ -72,6 +73,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.kvc_evict.argtypes = [vp, ctypes.c_int, p_i32, vp, vp]
     lib.kvc_attn_prefill_chunk.argtypes = [vp, ctypes.c_int, vp, vp, vp]
     lib.kvc_attn_decode.argtypes = [vp, ctypes.c_int, vp, vp, vp]
+    lib.kvc_attn_decode_noalloc.argtypes = [vp, ctypes.c_int, vp, vp, vp]
     lib.kvc_resident_size.argtypes = [vp, ctypes.c_int, ctypes.POINTER(i64)]
     lib.kvc_release.argtypes = [vp, ctypes.c_int, p_i32, vp]
     lib.kvc_export_state.argtypes = [vp, ctypes.c_int, ctypes.POINTER(SessionInfo), p_i32, p_i32,

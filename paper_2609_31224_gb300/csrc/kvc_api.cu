@@ -400,6 +400,25 @@ int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void*
   return KVC_OK;
 }
 
+int kvc_attn_decode_noalloc(kvc_ctx* ctx, int layer, const void* d_q, void* d_out,
+                            void* stream) {
+  g_err.clear();
+  int rc = check_attn(ctx, layer, d_q, d_out);
+  if (rc) return rc;
+  if (!ctx->last_single)
+    return fail(KVC_ESTATE, "decode needs exactly one appended token per session");
+  const int pairs = ctx->last_n_seq * ctx->cfg.kv_heads;
+  if (pairs > noalloc_max_pairs())
+    return fail(KVC_EINVAL,
+                "kvc_attn_decode_noalloc handles at most %d (session, kv-head) pairs per call; "
+                "this call has %d sessions x %d kv heads = %d",
+                noalloc_max_pairs(), ctx->last_n_seq, ctx->cfg.kv_heads, pairs);
+  const int cs = noalloc_chunks(ctx->d, ctx->last_n_seq);
+  KVC_CUDA(launch_attn_decode_noalloc(ctx->d, layer, d_q, d_out, ctx->last_n_seq, cs,
+                                      static_cast<cudaStream_t>(stream)));
+  return KVC_OK;
+}
+
 int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void* stream) {
   g_err.clear();
   int rc = check_attn(ctx, layer, d_q, d_out);

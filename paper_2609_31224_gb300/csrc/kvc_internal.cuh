@@ -273,6 +273,10 @@ cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                 int max_t, cudaStream_t s);
 int decode_grid_ctas(const Dev& d);
+int noalloc_max_pairs();
+int noalloc_chunks(const Dev& d, int n_seq);
+cudaError_t launch_attn_decode_noalloc(const Dev& d, int layer, const void* q, void* out,
+                                       int n_seq, int cs, cudaStream_t s);
 int prefill_grid_ctas(const Dev& d);
 
 }  // namespace kvc
