@@ -101,6 +101,12 @@ def _ptr_i32(a: np.ndarray):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
 
 
+def host_i32(a):
+    """(array, ctypes pointer) for a host int32 argument; keep the array alive."""
+    arr = _i32(a)
+    return arr, _ptr_i32(arr)
+
+
 def _stream(stream):
     import torch
     if stream is None:
@@ -151,6 +157,26 @@ class KVCache:
             self.close()
         except Exception:
             pass
+
+    # -- hot path, raw form: pointers and stream handle as Python ints ------------------
+    # For per-token loops where tensor indexing and stream lookup would dominate:
+    # ``sess_p`` / ``cu_p`` are ctypes int32 pointers (see ``host_i32``), the rest
+    # are device addresses and a cudaStream_t value.
+    def append_chunk_raw(self, n_seq, sess_p, cu_p, types_ptr, k_ptr, v_ptr, stream) -> None:
+        rc = self.lib.kvc_append_chunk(self.ctx, n_seq, sess_p, cu_p, types_ptr, k_ptr, v_ptr,
+                                       stream)
+        if rc:
+            _check(rc)
+
+    def attn_decode_raw(self, layer, q_ptr, out_ptr, stream) -> None:
+        rc = self.lib.kvc_attn_decode(self.ctx, layer, q_ptr, out_ptr, stream)
+        if rc:
+            _check(rc)
+
+    def attn_prefill_raw(self, layer, q_ptr, out_ptr, stream) -> None:
+        rc = self.lib.kvc_attn_prefill_chunk(self.ctx, layer, q_ptr, out_ptr, stream)
+        if rc:
+            _check(rc)
 
     # -- hot path -------------------------------------------------------------------
     def append_chunk(self, sessions, cu_tokens, types, k, v, stream=None) -> None:

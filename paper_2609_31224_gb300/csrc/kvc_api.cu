@@ -160,6 +160,7 @@ struct kvc_ctx {
   // Last append (queries of the following attention calls).
   bool attn_valid = false;
   int last_n_seq = 0, last_total = 0, last_max_t = 0;
+  int attn_since_append = 0;  // attention launches since the last append
   bool last_single = false;
   int dec_target = 0, pf_target = 0;
 };
@@ -335,6 +336,7 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, const i
   ctx->used_ub += need;
   ctx->delta_since_readback += need;
   ctx->attn_valid = true;
+  ctx->attn_since_append = 0;
   ctx->last_n_seq = n_seq;
   ctx->last_total = total;
   ctx->last_max_t = max_t;
@@ -395,8 +397,11 @@ int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void*
   if (rc) return rc;
   if (!ctx->last_single)
     return fail(KVC_ESTATE, "decode needs exactly one appended token per session");
+  // The first attention launch after an append follows the kernel that wrote the
+  // new token's K/V, so it does not start early; later ones may.
   KVC_CUDA(launch_attn_decode(ctx->d, layer, d_q, d_out, ctx->last_n_seq,
-                              static_cast<cudaStream_t>(stream)));
+                              ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream)));
+  ++ctx->attn_since_append;
   return KVC_OK;
 }
 
@@ -426,7 +431,8 @@ int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out
   if (ctx->last_max_t > PF_MAX_TOKENS)
     return fail(KVC_EINVAL, "prefill chunks are limited to %d tokens per session", PF_MAX_TOKENS);
   KVC_CUDA(launch_attn_prefill(ctx->d, layer, d_q, d_out, ctx->last_n_seq, ctx->last_max_t,
-                               static_cast<cudaStream_t>(stream)));
+                               ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream)));
+  ++ctx->attn_since_append;
   return KVC_OK;
 }
 

@@ -93,6 +93,11 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
   }
   if (tid == 0) s_abort = 0;
   __syncthreads();
+  // The next attention call may start its CTAs as soon as slots free up.  Before
+  // pdl_wait() this kernel reads only what the append wrote (work list, page
+  // tables, K/V pages); q, outputs, partials and counters come after it.
+  pdl_launch_dependents();
+  bool waited = false;
 
   const int n_items = d.g->n_dec_items * d.kv_heads;
   const size_t head_stride = (size_t)PS * D;  // elements between heads in a page
@@ -107,44 +112,58 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
     const int32_t* lrow = d.live_pt + (size_t)si.sid * d.max_pages_per_session;
     const int pos = si.pos_first;  // the single token of this session
 
-    // Query rows of the G heads, rotated at `pos`, scaled by log2(e)/sqrt(D).
-    float qr[G][C::VEC];
-    {
-      const T* qrow = q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G) * D;
-      const float2* cs = d.rope + (size_t)pos * (D / 2);
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-#pragma unroll
-        for (int e = 0; e < C::VEC; ++e) {
-          const int dd = c * C::VEC + e;
-          const bool lo = dd < D / 2;
-          const int j = lo ? dd : dd - D / 2;
-          const float x = to_float<T>(qrow[g * D + dd]);
-          const float y = to_float<T>(qrow[g * D + (lo ? dd + D / 2 : dd - D / 2)]);
-          const float2 t = cs[j];
-          const float r = lo ? fmaf(x, t.x, -y * t.y) : fmaf(x, t.x, y * t.y);
-          qr[g][e] = r * qk_scale;
-        }
-      }
-    }
-
     const int nblk = itm.blk_end - itm.blk_begin;
     const int n_my = (nblk > warp) ? (nblk - warp + DEC_WARPS - 1) / DEC_WARPS : 0;
+    // Page ids of this warp's blocks, 32 at a time: lane j holds block (win + j),
+    // so one round trip to the page table serves 32 loads.  Called warp-wide.
+    int pwin = -32, pid = 0;
     auto issue = [&](int k) {
-      const int b = itm.blk_begin + warp + k * DEC_WARPS;
-      const BlockRef br = block_ref(si, hrow, lrow, b);
-      const uint32_t n = loads + k;
-      const int st = n % STAGES;
-      uint8_t* dst = tiles + st * 2 * C::TILE;
-      const T* kp = reinterpret_cast<const T*>(d.pool) +
-                    pool_offset_elems(d, br.page, layer, 0, head, 0);
-      mbar_arrive_expect_tx(&wbars[st], 2 * C::TILE);
-      bulk_g2s(dst, kp, C::TILE, &wbars[st]);
-      bulk_g2s(dst + C::TILE, kp + d.kv_heads * head_stride, C::TILE, &wbars[st]);
+      if (k >= pwin + 32) {
+        pwin = k & ~31;
+        const int j = pwin + lane;
+        pid = j < n_my ? block_page(si, hrow, lrow, itm.blk_begin + warp + j * DEC_WARPS) : 0;
+      }
+      const int page = __shfl_sync(FULL, pid, k - pwin);
+      if (lane == 0) {
+        const uint32_t n = loads + k;
+        const int st = n % STAGES;
+        uint8_t* dst = tiles + st * 2 * C::TILE;
+        const T* kp = reinterpret_cast<const T*>(d.pool) +
+                      pool_offset_elems(d, page, layer, 0, head, 0);
+        mbar_arrive_expect_tx(&wbars[st], 2 * C::TILE);
+        bulk_g2s(dst, kp, C::TILE, &wbars[st]);
+        bulk_g2s(dst + C::TILE, kp + d.kv_heads * head_stride, C::TILE, &wbars[st]);
+      }
     };
-    if (lane == 0) {
-      fence_proxy_async_smem();  // the stage buffers were written by the previous merge
-      for (int k = 0; k < min(STAGES, n_my); ++k) issue(k);
+    // The stage buffers were written by the previous merge: fence before TMA reuse.
+    if (lane == 0) fence_proxy_async_smem();
+    for (int k = 0; k < min(STAGES, n_my); ++k) issue(k);
+
+    if (!waited) {
+      pdl_wait();
+      waited = true;
+    }
+    // Query rows of the G heads, rotated at `pos`, scaled by log2(e)/sqrt(D).  Lane c
+    // holds 16-byte chunk c of each row; its rotate-half partner is chunk c ^ 8.
+    float qr[G][C::VEC];
+    {
+      const uint8_t* qrow = reinterpret_cast<const uint8_t*>(
+          q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G) * D);
+      const float2* cs = d.rope + (size_t)pos * (D / 2) + (c & 7) * C::VEC;
+      const bool lo = c < 8;
+      float2 t[C::VEC];
+#pragma unroll
+      for (int e = 0; e < C::VEC; ++e) t[e] = cs[e];
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        float x[C::VEC], y[C::VEC];
+        load_vec<T>(qrow + g * C::ROW_BYTES + c * 16, x);
+        load_vec<T>(qrow + g * C::ROW_BYTES + (c ^ 8) * 16, y);
+#pragma unroll
+        for (int e = 0; e < C::VEC; ++e)
+          qr[g][e] = (lo ? fmaf(x[e], t[e].x, -y[e] * t[e].y) : fmaf(x[e], t[e].x, y[e] * t[e].y)) *
+                     qk_scale;
+      }
     }
 
     float m_run = -INFINITY, l_run = 0.f;  // for row g_sm = lane >> 3
@@ -159,14 +178,13 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
       const uint32_t n = loads + k;
       const int st = n % STAGES;
       const uint32_t parity = (n / STAGES) & 1;
-      if (!mbar_wait(d, &wbars[st], parity)) {
+      if (!__all_sync(FULL, mbar_wait(d, &wbars[st], parity))) {
         failed_at = k;
         break;
       }
       const uint8_t* kt = tiles + st * 2 * C::TILE;
       const uint8_t* vt = kt + C::TILE;
-      const int b = itm.blk_begin + warp + k * DEC_WARPS;
-      const BlockRef br = block_ref(si, hrow, lrow, b);
+      const BlockRange br = block_range(si, itm.blk_begin + warp + k * DEC_WARPS);
 
       // Scores: lanes 0-15 take even keys, 16-31 odd keys; each lane a 16-byte chunk.
 #pragma unroll
@@ -243,8 +261,8 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
         }
       }
       __syncwarp();
-      if (lane == 0 && k + STAGES < n_my) {
-        fence_proxy_async_smem();
+      if (k + STAGES < n_my) {
+        if (lane == 0) fence_proxy_async_smem();
         issue(k + STAGES);
       }
     }
@@ -335,23 +353,39 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
           for (int ch = lane; ch < nch; ch += 32) s_scale[ch * G + g] *= inv;
         }
         __syncthreads();
-        for (int e = tid; e < G * D; e += DEC_THREADS) {
-          const int g = e / D, dd = e % D;
-          float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
-          int ch = 0;
-          for (; ch + 4 <= nch; ch += 4) {
-            const size_t b0 = ((size_t)(s0 + ch * d.kv_heads) * G + g) * D + dd;
-            const size_t st = (size_t)d.kv_heads * G * D;
-            O0 += __ldcg(&d.dec_part_o[b0]) * s_scale[ch * G + g];
-            O1 += __ldcg(&d.dec_part_o[b0 + st]) * s_scale[(ch + 1) * G + g];
-            O2 += __ldcg(&d.dec_part_o[b0 + 2 * st]) * s_scale[(ch + 2) * G + g];
-            O3 += __ldcg(&d.dec_part_o[b0 + 3 * st]) * s_scale[(ch + 3) * G + g];
+        // Each thread owns EPT output elements; per chunk it issues their loads
+        // together (two chunks per iteration), so many loads are in flight.
+        constexpr int EPT = G * D / DEC_THREADS;
+        const size_t cstride = (size_t)d.kv_heads * G * D;
+        const float* base = d.dec_part_o + (size_t)s0 * G * D;
+        float O[EPT];
+#pragma unroll
+        for (int i = 0; i < EPT; ++i) O[i] = 0.f;
+        int ch = 0;
+        for (; ch + 2 <= nch; ch += 2) {
+          float a0[EPT], a1[EPT];
+#pragma unroll
+          for (int i = 0; i < EPT; ++i) {
+            a0[i] = __ldcg(base + ch * cstride + tid + i * DEC_THREADS);
+            a1[i] = __ldcg(base + (ch + 1) * cstride + tid + i * DEC_THREADS);
           }
-          for (; ch < nch; ++ch)
-            O0 += __ldcg(&d.dec_part_o[((size_t)(s0 + ch * d.kv_heads) * G + g) * D + dd]) *
-                  s_scale[ch * G + g];
-          out[((size_t)si.q_row0 * d.q_heads + head * G + g) * D + dd] =
-              from_float<T>((O0 + O1) + (O2 + O3));
+#pragma unroll
+          for (int i = 0; i < EPT; ++i) {
+            const int g = (tid + i * DEC_THREADS) / D;
+            O[i] += a0[i] * s_scale[ch * G + g] + a1[i] * s_scale[(ch + 1) * G + g];
+          }
+        }
+        for (; ch < nch; ++ch) {
+#pragma unroll
+          for (int i = 0; i < EPT; ++i) {
+            const int g = (tid + i * DEC_THREADS) / D;
+            O[i] += __ldcg(base + ch * cstride + tid + i * DEC_THREADS) * s_scale[ch * G + g];
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < EPT; ++i) {
+          const int e = tid + i * DEC_THREADS;
+          out[((size_t)si.q_row0 * d.q_heads + head * G) * D + e] = from_float<T>(O[i]);
         }
         if (tid == 0) d.dec_count[itm.seq * d.kv_heads + head] = 0;
       }
@@ -387,22 +421,20 @@ int decode_grid_ctas(const Dev& d) {
 }
 
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               cudaStream_t s) {
+                               bool pdl, cudaStream_t s) {
   (void)n_seq;
   static thread_local int grid_bf16 = 0, grid_f32 = 0;
   const float scale = LOG2E / sqrtf((float)d.head_dim);
   if (d.esz == 2) {
     if (!grid_bf16) grid_bf16 = decode_grid_ctas(d);
-    attn_decode_kernel<__nv_bfloat16, 128, DEC_STAGES>
-        <<<grid_bf16, DEC_THREADS, dec_smem<__nv_bfloat16, 128>(), s>>>(
-            d, layer, static_cast<const __nv_bfloat16*>(q), static_cast<__nv_bfloat16*>(out),
-            scale);
-  } else {
-    if (!grid_f32) grid_f32 = decode_grid_ctas(d);
-    attn_decode_kernel<float, 64, DEC_STAGES><<<grid_f32, DEC_THREADS, dec_smem<float, 64>(), s>>>(
-        d, layer, static_cast<const float*>(q), static_cast<float*>(out), scale);
+    return launch_ex(&attn_decode_kernel<__nv_bfloat16, 128, DEC_STAGES>, dim3(grid_bf16),
+                     dim3(DEC_THREADS), dec_smem<__nv_bfloat16, 128>(), s, pdl, d, layer,
+                     static_cast<const __nv_bfloat16*>(q), static_cast<__nv_bfloat16*>(out), scale);
   }
-  return cudaGetLastError();
+  if (!grid_f32) grid_f32 = decode_grid_ctas(d);
+  return launch_ex(&attn_decode_kernel<float, 64, DEC_STAGES>, dim3(grid_f32), dim3(DEC_THREADS),
+                   dec_smem<float, 64>(), s, pdl, d, layer, static_cast<const float*>(q),
+                   static_cast<float*>(out), scale);
 }
 
 }  // namespace kvc

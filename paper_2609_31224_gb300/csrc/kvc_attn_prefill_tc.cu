@@ -1,0 +1,618 @@
+// Chunked-prefill GQA attention on the 5th-generation tensor cores (tcgen05 +
+// TMEM), bfloat16 K/V/q, fp32 softmax and accumulation.
+//
+// Per work item (session, KV head, chunk of resident pages) the T*G query rows
+// (T <= 32 tokens, G = 4 heads) form the M = 128 rows of an MMA tile; the
+// rows past T*G are zero padding.  Warp roles in one CTA:
+//   warp 0    producer: 2-D TMA loads (128-byte swizzle) of 4 K/V pages
+//             (64 keys) per stage into a shared-memory ring;
+//   warp 1    MMA issuer: one elected thread issues tcgen05.mma from
+//             shared-memory descriptors, S = Q K^T (N = 64) into a
+//             double-buffered TMEM tile and O += P V (N = 128) into TMEM;
+//             completion is signalled with tcgen05.commit on mbarriers;
+//   warps 2-5 softmax: each thread owns one TMEM lane (= one query row):
+//             it builds its rotated, scaled query row in shared memory,
+//             reads its row of S from TMEM, masks (resident slots, causal
+//             inside the chunk), keeps the running max/sum, writes P as
+//             bfloat16 to a swizzled shared buffer, rescales O in TMEM when
+//             the row maximum grows by more than 2^8, and finally reads O.
+// All waits are bounded; a timeout records KVC_DERR_WAIT and the CTA stops.
+#include <cuda.h>
+
+#include "kvc_internal.cuh"
+
+namespace kvc {
+
+namespace {
+
+constexpr int G = 4;
+constexpr int D = 128;
+constexpr int M = 128;                       // MMA rows (query rows, padded)
+constexpr int NK = 64;                       // keys per stage (4 pages)
+constexpr int TC_STAGES = 4;                 // K/V stages
+constexpr int KV_PANEL = NK * 128;           // 64 rows x 128 B = 8 KiB
+constexpr int STAGE = 4 * KV_PANEL;          // K lo, K hi, V lo, V hi = 32 KiB
+constexpr int Q_PANEL = M * 128;             // 16 KiB
+constexpr int Q_BYTES = 2 * Q_PANEL;         // 32 KiB
+constexpr int P_BYTES = M * 128;             // 128 rows x 64 keys bf16 = 16 KiB
+constexpr int TMEM_COLS = 256;               // S0 [0,64) S1 [64,128) O [128,256)
+constexpr int S_COL = 0, O_COL = 128;
+constexpr float LOG2E = 1.4426950408889634f;
+constexpr float RESCALE_LOG2 = 8.f;          // rescale O only when the max grows by > 2^8
+constexpr int THREADS = 6 * 32;
+constexpr unsigned FULL = 0xFFFFFFFFu;
+
+// Shared memory map (offsets from a 1024-aligned base).
+constexpr int OFF_Q = 0;
+constexpr int OFF_KV = OFF_Q + Q_BYTES;
+constexpr int OFF_P = OFF_KV + TC_STAGES * STAGE;
+constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+enum {
+  B_KV_FULL = 0,                         // [TC_STAGES]
+  B_KV_EMPTY = B_KV_FULL + TC_STAGES,    // [TC_STAGES]
+  B_S_FULL = B_KV_EMPTY + TC_STAGES,     // [2]
+  B_S_EMPTY = B_S_FULL + 2,              // [2]
+  B_P_FULL = B_S_EMPTY + 2,              // [2]
+  B_P_EMPTY = B_P_FULL + 2,              // [2]
+  B_O = B_P_EMPTY + 2,                   // one phase per P V product
+  B_Q = B_O + 1,                         // one phase per item (query tile ready)
+  B_FINAL = B_Q + 1,                     // every MMA of the CTA complete
+  N_BARS = B_FINAL + 1
+};
+constexpr int OFF_TMEM_ADDR = OFF_BAR + N_BARS * 8;
+constexpr int TC_SMEM = OFF_TMEM_ADDR + 16 + 1024;  // + alignment slack
+
+// -- tcgen05 helpers ------------------------------------------------------------------
+__device__ inline void tmem_alloc(uint32_t* smem_dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(smem_dst)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ inline void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ inline void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ inline void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ inline void tc_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+__device__ inline void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                              uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Each thread of the warp reads 32 consecutive fp32 columns of its TMEM lane.
+__device__ inline void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ inline void tmem_st32(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+      "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
+          taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle: `sbo` bytes between 8-row
+// groups; `lbo` bytes between 64-element groups of the contiguous dimension
+// (MN-major operands only).
+__device__ inline uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFF);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+  d |= (uint64_t)1 << 46;  // descriptor version of this architecture
+  d |= (uint64_t)2 << 61;  // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major, B K- or MN-major.
+__host__ __device__ constexpr uint32_t instr_desc(int n, int m, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ inline void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y,
+                                   uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ inline uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ inline float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// 16-byte chunk `c` (0..7) of row `r` of a 128-byte-swizzled panel.
+__device__ inline uint32_t sw128(uint32_t panel, int r, int c) {
+  return panel + r * 128 + ((c ^ (r & 7)) << 4);
+}
+
+__device__ inline void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                    uint32_t e) {
+  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+               "r"(e)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
+    Dev d, int layer, const __grid_constant__ CUtensorMap map_lo,
+    const __grid_constant__ CUtensorMap map_hi, const __nv_bfloat16* __restrict__ q,
+    __nv_bfloat16* __restrict__ out, float qk_scale) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_TMEM_ADDR);
+  __shared__ int s_abort_flag, s_last;
+  volatile int& s_abort = s_abort_flag;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+  if (tid == 0) {
+    for (int s = 0; s < TC_STAGES; ++s) {
+      mbar_init(&bars[B_KV_FULL + s], 1);
+      mbar_init(&bars[B_KV_EMPTY + s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bars[B_S_FULL + s], 1);
+      mbar_init(&bars[B_S_EMPTY + s], 4);
+      mbar_init(&bars[B_P_FULL + s], 4);
+      mbar_init(&bars[B_P_EMPTY + s], 1);
+    }
+    mbar_init(&bars[B_O], 1);
+    mbar_init(&bars[B_Q], 4);
+    mbar_init(&bars[B_FINAL], 1);
+    fence_mbar_init();
+    s_abort = 0;
+  }
+  // Zero the query, K/V and P tiles once: padding query rows stay zero, and the
+  // keys of partly filled stages only ever hold finite values (their weights are
+  // 0, and 0 times a stale NaN would not be 0).
+  for (int i = tid; i < OFF_BAR / 16; i += THREADS)
+    reinterpret_cast<uint4*>(smem)[i] = make_uint4(0, 0, 0, 0);
+  fence_proxy_async_smem();
+  if (warp == 1) tmem_alloc(tmem_slot, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  // Before pdl_wait() only the append's data is read (work list, page tables, K/V
+  // pages); the softmax warps wait before reading q or writing any result.
+  pdl_launch_dependents();
+
+  const int H = d.kv_heads, L = d.layers;
+  const int n_items = d.g->n_pf_items * H;
+  const uint32_t sQ = smem_u32(smem + OFF_Q);
+  const uint32_t sKV = smem_u32(smem + OFF_KV);
+  const uint32_t sP = smem_u32(smem + OFF_P);
+
+  if (warp == 0) {
+    // ---------------- producer ----------------
+    // The whole warp walks the items; lane j fetches the page id of block
+    // (window + j) so that one round trip serves 32 blocks, and lane 0 issues the
+    // TMA loads with the ids shuffled to it.
+    uint32_t n = 0;  // stages produced
+    bool stop = false;
+    for (int it = blockIdx.x; it < n_items && !stop; it += gridDim.x) {
+      const int item = it / H, head = it % H;
+      const Item itm = d.pf_items[item];
+      const SeqInfo si = d.seq[itm.seq];
+      const int32_t* hrow = d.hist_pt + (size_t)si.sid * d.max_pages_per_session;
+      const int32_t* lrow = d.live_pt + (size_t)si.sid * d.max_pages_per_session;
+      const int nblk = itm.blk_end - itm.blk_begin;
+      const int n_st = (nblk + 3) / 4;
+      int pid = 0;
+      for (int k = 0; k < n_st; ++k, ++n) {
+        const int b0 = 4 * k;
+        if ((b0 & 31) == 0) {
+          const int bj = b0 + lane;
+          pid = bj < nblk ? block_page(si, hrow, lrow, itm.blk_begin + bj) : 0;
+        }
+        const int st = n % TC_STAGES;
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait(d, &bars[B_KV_EMPTY + st], ((n / TC_STAGES) & 1) ^ 1);
+        ok = __shfl_sync(FULL, ok, 0);
+        if (!ok) {
+          if (lane == 0) s_abort = 1;
+          stop = true;
+          break;
+        }
+        const int npg = min(4, nblk - b0);
+        int pages[4];
+#pragma unroll
+        for (int pg = 0; pg < 4; ++pg) pages[pg] = __shfl_sync(FULL, pid, (b0 & 31) + pg);
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&bars[B_KV_FULL + st], npg * 4 * 2048);
+          uint8_t* base = smem + OFF_KV + st * STAGE;
+          for (int pg = 0; pg < npg; ++pg) {
+            const int rk = (((pages[pg] * L + layer) * 2 + 0) * H + head) * PS;
+            const int rv = rk + H * PS;
+            tma_load_2d(base + 0 * KV_PANEL + pg * 2048, &map_lo, 0, rk, &bars[B_KV_FULL + st]);
+            tma_load_2d(base + 1 * KV_PANEL + pg * 2048, &map_hi, 0, rk, &bars[B_KV_FULL + st]);
+            tma_load_2d(base + 2 * KV_PANEL + pg * 2048, &map_lo, 0, rv, &bars[B_KV_FULL + st]);
+            tma_load_2d(base + 3 * KV_PANEL + pg * 2048, &map_hi, 0, rv, &bars[B_KV_FULL + st]);
+          }
+        }
+      }
+      stop = stop || __any_sync(FULL, s_abort != 0);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t ID_S = instr_desc(NK, M, false);
+      constexpr uint32_t ID_PV = instr_desc(D, M, true);
+      uint32_t n = 0;      // K/V stages consumed
+      uint32_t sc = 0;     // S tiles issued
+      uint32_t pv = 0;     // P V products issued
+      uint32_t items = 0;  // items started
+      for (int it = blockIdx.x; it < n_items && !s_abort; it += gridDim.x, ++items) {
+        const Item itm = d.pf_items[it / H];
+        const int nblk = itm.blk_end - itm.blk_begin;
+        const int n_st = (nblk + 3) / 4;
+        if (!mbar_wait(d, &bars[B_Q], items & 1)) {
+          s_abort = 1;
+          break;
+        }
+        tc_fence_after();
+        // S(k) is issued before P(k-1) V(k-1) so the softmax of stage k overlaps it.
+        for (int k = 0; k <= n_st && !s_abort; ++k) {
+          if (k < n_st) {
+            const int st = (n + k) % TC_STAGES;
+            const int sb = sc % 2;
+            if (!mbar_wait(d, &bars[B_KV_FULL + st], ((n + k) / TC_STAGES) & 1) ||
+                !mbar_wait(d, &bars[B_S_EMPTY + sb], ((sc / 2) & 1) ^ 1)) {
+              s_abort = 1;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t kbase = sKV + st * STAGE;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t qa = sQ + (kk >> 2) * Q_PANEL + (kk & 3) * 32;
+              const uint32_t kb = kbase + (kk >> 2) * KV_PANEL + (kk & 3) * 32;
+              tc_mma(tmem + S_COL + sb * NK, smem_desc(qa, 0, 1024), smem_desc(kb, 0, 1024),
+                     ID_S, kk > 0 ? 1u : 0u);
+            }
+            tc_commit(&bars[B_S_FULL + sb]);
+            ++sc;
+          }
+          if (k >= 1) {
+            const int kp = k - 1;
+            const int st = (n + kp) % TC_STAGES;
+            const int pb = pv % 2;
+            if (!mbar_wait(d, &bars[B_P_FULL + pb], (pv / 2) & 1)) {
+              s_abort = 1;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t vbase = sKV + st * STAGE + 2 * KV_PANEL;
+            const uint32_t pbase = sP + pb * P_BYTES;
+#pragma unroll
+            for (int kk = 0; kk < NK / 16; ++kk) {
+              const uint32_t pa = pbase + kk * 32;
+              const uint32_t vb = vbase + kk * 16 * 128;
+              tc_mma(tmem + O_COL, smem_desc(pa, 0, 1024), smem_desc(vb, KV_PANEL, 1024), ID_PV,
+                     (kp > 0 || kk > 0) ? 1u : 0u);
+            }
+            tc_commit(&bars[B_KV_EMPTY + st]);
+            tc_commit(&bars[B_P_EMPTY + pb]);
+            tc_commit(&bars[B_O]);
+            ++pv;
+          }
+        }
+        n += n_st;
+      }
+      // No MMA may still be running when the tensor memory is released.
+      tc_commit(&bars[B_FINAL]);
+      mbar_wait(d, &bars[B_FINAL], 0);
+    }
+  } else {
+    // ---------------- softmax / epilogue ----------------
+    // A failed (timed-out) wait makes the warp "dead": it then skips waits and
+    // work but still walks the same items, arrivals and named barriers, so the
+    // other softmax warps never wait for it.
+    const int quarter = warp & 3;              // TMEM lanes 32*quarter .. +31
+    const int r = quarter * 32 + lane;         // this thread's query row
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    uint32_t sc = 0, pv = 0;
+    bool dead = false;
+    pdl_wait();
+    auto wait = [&](uint64_t* bar, uint32_t parity) {
+      if (dead) return;
+      dead = !__all_sync(FULL, mbar_wait(d, bar, parity));
+      if (dead && lane == 0) s_abort = 1;
+    };
+    for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
+      const int item = it / H, head = it % H;
+      const Item itm = d.pf_items[item];
+      const SeqInfo si = d.seq[itm.seq];
+      const int32_t* hrow = d.hist_pt + (size_t)si.sid * d.max_pages_per_session;
+      const int32_t* lrow = d.live_pt + (size_t)si.sid * d.max_pages_per_session;
+      const int nblk = itm.blk_end - itm.blk_begin;
+      const int n_st = (nblk + 3) / 4;
+      const int R = si.t * G;
+      const bool live = r < R;
+      const int t = r / G, g = r % G;
+      const int qlog = si.n_hist + si.n_live - si.t + t;
+      // The previous item's products are complete (its epilogue waited for the
+      // last one), so the query tile can be overwritten.
+      if (live && !dead) {
+        // Chunk c (dims 8c..8c+7) of the first half pairs with chunk c of the second.
+        const uint4* qrow = reinterpret_cast<const uint4*>(
+            q + ((size_t)(si.q_row0 + t) * d.q_heads + head * G + g) * D);
+        const float4* cs = reinterpret_cast<const float4*>(d.rope + (size_t)(si.pos_first + t) * (D / 2));
+#pragma unroll 2
+        for (int c = 0; c < 8; ++c) {
+          const uint4 wa = qrow[c], wb = qrow[c + 8];
+          const uint32_t ua[4] = {wa.x, wa.y, wa.z, wa.w}, ub[4] = {wb.x, wb.y, wb.z, wb.w};
+          float ya[8], yb[8];
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const float4 t4 = cs[c * 4 + h];  // (cos, sin) of dims 8c + 2h, 8c + 2h + 1
+            const float a0 = bf16lo(ua[h]), a1 = bf16hi(ua[h]);
+            const float b0 = bf16lo(ub[h]), b1 = bf16hi(ub[h]);
+            ya[2 * h] = fmaf(a0, t4.x, -b0 * t4.y) * qk_scale;
+            yb[2 * h] = fmaf(b0, t4.x, a0 * t4.y) * qk_scale;
+            ya[2 * h + 1] = fmaf(a1, t4.z, -b1 * t4.w) * qk_scale;
+            yb[2 * h + 1] = fmaf(b1, t4.z, a1 * t4.w) * qk_scale;
+          }
+          st_shared_v4(sw128(sQ, r, c), pack_bf16(ya[0], ya[1]), pack_bf16(ya[2], ya[3]),
+                       pack_bf16(ya[4], ya[5]), pack_bf16(ya[6], ya[7]));
+          st_shared_v4(sw128(sQ + Q_PANEL, r, c), pack_bf16(yb[0], yb[1]), pack_bf16(yb[2], yb[3]),
+                       pack_bf16(yb[4], yb[5]), pack_bf16(yb[6], yb[7]));
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars[B_Q]);
+
+      float m_used = -INFINITY, l = 0.f;
+      for (int k = 0; k < n_st; ++k) {
+        const int sb = sc % 2, pb = pv % 2;
+        wait(&bars[B_S_FULL + sb], (sc / 2) & 1);
+        tc_fence_after();
+        float s[NK];
+        tmem_ld32(trow + S_COL + sb * NK, s);
+        tmem_ld32(trow + S_COL + sb * NK + 32, s + 32);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_S_EMPTY + sb]);
+        ++sc;
+        // Mask the keys that are not resident slots or lie after the row's query.
+        // Interior stages (four full pages, every key before the chunk's first
+        // query) need no mask.  Padding rows (r >= T*G) are left unmasked: their
+        // products stay finite and their outputs are never written.
+        const int npg = min(4, nblk - 4 * k);
+        BlockRange brs[4];
+        bool interior = npg == 4;
+#pragma unroll
+        for (int pg = 0; pg < 4; ++pg) {
+          brs[pg] = block_range(si, itm.blk_begin + 4 * k + min(pg, npg - 1));
+          interior = interior && brs[pg].lo == 0 && brs[pg].hi == PS;
+        }
+        interior = interior && brs[3].base + PS - 1 <= si.n_hist + si.n_live - si.t;
+        if (!interior) {
+#pragma unroll
+          for (int pg = 0; pg < 4; ++pg) {
+#pragma unroll
+            for (int j = 0; j < PS; ++j) {
+              const bool v = pg < npg && j >= brs[pg].lo && j < brs[pg].hi &&
+                             brs[pg].base + j <= qlog;
+              float& x = s[pg * PS + j];
+              x = (v || !live) ? x : -INFINITY;
+            }
+          }
+        }
+        float mx = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < NK; ++j) mx = fmaxf(mx, s[j]);
+        if (dead || !live) mx = -INFINITY;
+        // Rescale O (in TMEM) and l only when the row maximum grows by > 2^8; this
+        // waits for the previous P V product.  Every lane of the warp takes part
+        // in the TMEM accesses; lanes that need no rescale use factor 1.
+        const bool need = mx > m_used + RESCALE_LOG2;
+        const bool have_o = pv > 0 && m_used != -INFINITY;
+        if (__any_sync(FULL, need && have_o)) {
+          wait(&bars[B_O], (pv - 1) & 1);
+          tc_fence_after();
+          const float f = (need && have_o) ? exp2f(m_used - mx) : 1.f;
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld32(trow + O_COL + c * 32, o);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= f;
+            tmem_st32(trow + O_COL + c * 32, o);
+          }
+          tc_fence_before();
+        }
+        if (need) {
+          if (have_o) l *= exp2f(m_used - mx);
+          m_used = mx;
+        }
+        // P = exp2(s - m_used) as bfloat16 into P buffer pb (row r, 64 keys = 128 B).
+        wait(&bars[B_P_EMPTY + pb], ((pv / 2) & 1) ^ 1);
+        // Masked keys are -inf and give 0; a row with no finite key yet uses 0 as
+        // its reference so that no -inf - -inf appears; padding rows get weight 0.
+        const float mref = !live ? INFINITY : (m_used == -INFINITY ? 0.f : m_used);
+        float rs0 = 0.f, rs1 = 0.f;
+        uint32_t pw[NK / 2];
+#pragma unroll
+        for (int j = 0; j < NK; j += 2) {
+          const float p0 = ex2(s[j] - mref), p1 = ex2(s[j + 1] - mref);
+          rs0 += p0;
+          rs1 += p1;
+          pw[j / 2] = pack_bf16(p0, p1);
+        }
+        l += rs0 + rs1;
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          st_shared_v4(sw128(sP + pb * P_BYTES, r, c), pw[4 * c], pw[4 * c + 1], pw[4 * c + 2],
+                       pw[4 * c + 3]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_P_FULL + pb]);
+        ++pv;
+      }
+      // Epilogue: wait for the last P V, read O.
+      wait(&bars[B_O], (pv - 1) & 1);
+      tc_fence_after();
+      const bool single = si.pf_chunks == 1;
+      const int slot = (si.pf_base + itm.chunk) * H + head;
+      const size_t prow0 = (size_t)slot * (PF_MAX_TOKENS * G) + r;
+      const bool write = live && !dead;
+      const float inv = 1.f / l;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        float o[32];
+        tmem_ld32(trow + O_COL + c * 32, o);
+        if (write && single) {
+          __nv_bfloat16* orow =
+              out + ((size_t)(si.q_row0 + t) * d.q_heads + head * G + g) * D + c * 32;
+#pragma unroll
+          for (int i = 0; i < 32; i += 8)
+            *reinterpret_cast<uint4*>(orow + i) =
+                make_uint4(pack_bf16(o[i] * inv, o[i + 1] * inv),
+                           pack_bf16(o[i + 2] * inv, o[i + 3] * inv),
+                           pack_bf16(o[i + 4] * inv, o[i + 5] * inv),
+                           pack_bf16(o[i + 6] * inv, o[i + 7] * inv));
+        } else if (write) {
+          float* prow = d.pf_part_o + prow0 * D + c * 32;
+#pragma unroll
+          for (int i = 0; i < 32; i += 4)
+            *reinterpret_cast<float4*>(prow + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
+        }
+      }
+      tc_fence_before();
+      if (!single) {
+        // Split-K: publish this chunk's (O, max, sum); the last CTA to arrive for the
+        // (session, head) merges every chunk, one thread per query row.  All four
+        // softmax warps reach both named barriers on every such item.
+        if (write) d.pf_part_ml[prow0] = make_float2(m_used, l);
+        __threadfence();
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (warp == 2 && lane == 0) {
+          const int old = atomicAdd(&d.pf_count[itm.seq * H + head], 1);
+          s_last = (old == si.pf_chunks - 1);
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (s_last) {
+          __threadfence();
+          if (live) {
+            const size_t s0 = (size_t)(si.pf_base * H + head) * (PF_MAX_TOKENS * G) + r;
+            const size_t cstride = (size_t)H * (PF_MAX_TOKENS * G);
+            float Mx = -INFINITY;
+            for (int ch = 0; ch < si.pf_chunks; ++ch)
+              Mx = fmaxf(Mx, __ldcg(&d.pf_part_ml[s0 + ch * cstride]).x);
+            float Ls = 0.f;
+            for (int ch = 0; ch < si.pf_chunks; ++ch) {
+              const float2 ml = __ldcg(&d.pf_part_ml[s0 + ch * cstride]);
+              Ls += ml.y * exp2_safe(ml.x, Mx);
+            }
+            const float invL = 1.f / Ls;
+            __nv_bfloat16* orow =
+                out + ((size_t)(si.q_row0 + t) * d.q_heads + head * G + g) * D;
+            for (int c = 0; c < D / 32; ++c) {
+              float acc[32];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+              for (int ch = 0; ch < si.pf_chunks; ++ch) {
+                const size_t row = s0 + ch * cstride;
+                const float sc2 = exp2_safe(__ldcg(&d.pf_part_ml[row]).x, Mx) * invL;
+                const float4* src =
+                    reinterpret_cast<const float4*>(d.pf_part_o + row * D + c * 32);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                  const float4 v = __ldcg(src + i);
+                  acc[4 * i] += v.x * sc2;
+                  acc[4 * i + 1] += v.y * sc2;
+                  acc[4 * i + 2] += v.z * sc2;
+                  acc[4 * i + 3] += v.w * sc2;
+                }
+              }
+#pragma unroll
+              for (int i = 0; i < 32; i += 8)
+                *reinterpret_cast<uint4*>(orow + c * 32 + i) =
+                    make_uint4(pack_bf16(acc[i], acc[i + 1]), pack_bf16(acc[i + 2], acc[i + 3]),
+                               pack_bf16(acc[i + 4], acc[i + 5]),
+                               pack_bf16(acc[i + 6], acc[i + 7]));
+            }
+          }
+          if (warp == 2 && lane == 0) d.pf_count[itm.seq * H + head] = 0;
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, TMEM_COLS);
+}
+
+}  // namespace
+
+const void* prefill_tc_kernel_ptr() {
+  return reinterpret_cast<const void*>(&attn_prefill_tc_kernel);
+}
+int prefill_tc_smem() { return TC_SMEM; }
+int prefill_tc_threads() { return THREADS; }
+
+cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,
+                                   const CUtensorMap& hi, const void* q, void* out, int grid,
+                                   bool pdl, cudaStream_t s) {
+  const float scale = LOG2E / sqrtf((float)d.head_dim);
+  return launch_ex(&attn_prefill_tc_kernel, dim3(grid), dim3(THREADS), TC_SMEM, s, pdl, d, layer,
+                   lo, hi, static_cast<const __nv_bfloat16*>(q), static_cast<__nv_bfloat16*>(out),
+                   scale);
+}
+
+}  // namespace kvc

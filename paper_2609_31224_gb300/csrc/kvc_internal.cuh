@@ -2,6 +2,7 @@
 // the PTX helpers (mbarrier, bulk copy) the kernels share.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -144,6 +145,32 @@ __device__ inline BlockRef block_ref(const SeqInfo& si, const int32_t* hist_row,
   return r;
 }
 
+// Valid slot range [lo, hi) and logical base of virtual block b, without
+// touching memory (the page id is looked up separately, see block_page).
+struct BlockRange {
+  int lo, hi, base;
+};
+
+__device__ inline BlockRange block_range(const SeqInfo& si, int b) {
+  BlockRange r;
+  if (b < si.n_hist_pages) {
+    r.lo = 0;
+    r.hi = min(PS, si.n_hist - b * PS);
+    r.base = b * PS;
+  } else {
+    const int s0 = (b - si.n_hist_pages) * PS;
+    r.lo = max(0, si.live_head - s0);
+    r.hi = min(PS, si.live_head + si.n_live - s0);
+    r.base = si.n_hist + s0 - si.live_head;
+  }
+  return r;
+}
+
+__device__ inline int block_page(const SeqInfo& si, const int32_t* hist_row,
+                                 const int32_t* live_row, int b) {
+  return b < si.n_hist_pages ? hist_row[b] : live_row[b - si.n_hist_pages];
+}
+
 __device__ inline void set_error(const Dev& d, int bits) { atomicOr(&d.g->err, bits); }
 
 // ---------------------------------------------------------------------------
@@ -213,6 +240,30 @@ __device__ inline void bulk_g2s(void* dst_smem, const void* src_gmem, uint32_t b
       : "memory");
 }
 
+// Programmatic dependent launch: let the next kernel in the stream start its
+// CTAs early, and wait until the previous kernel's writes are visible.
+__device__ inline void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ inline void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Launch with an optional programmatic-stream-serialization attribute.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t s, bool pdl, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // ---------------------------------------------------------------------------
 // Small numeric helpers.
 // ---------------------------------------------------------------------------
@@ -269,10 +320,16 @@ cudaError_t launch_append(const Dev& d, const AppendArgs& a, const uint8_t* type
 cudaError_t launch_evict(const Dev& d, const SeqArgs& a, int64_t* resident_out, cudaStream_t s);
 cudaError_t launch_release(const Dev& d, const SeqArgs& a, cudaStream_t s);
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               cudaStream_t s);
+                               bool pdl, cudaStream_t s);
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                                int max_t, cudaStream_t s);
+                                int max_t, bool pdl, cudaStream_t s);
 int decode_grid_ctas(const Dev& d);
+cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,
+                                   const CUtensorMap& hi, const void* q, void* out, int grid,
+                                   bool pdl, cudaStream_t s);
+const void* prefill_tc_kernel_ptr();
+int prefill_tc_smem();
+int prefill_tc_threads();
 int noalloc_max_pairs();
 int noalloc_chunks(const Dev& d, int n_seq);
 cudaError_t launch_attn_decode_noalloc(const Dev& d, int layer, const void* q, void* out,

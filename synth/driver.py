@@ -66,6 +66,7 @@ class Call:
     v: object = None
     q: object = None               # device [L][total][Hq][D]
     out: object = None             # device [total][Hq][D]
+    raw: tuple = None              # host pointers / device addresses for the raw calls
 
 
 @dataclass
@@ -95,6 +96,7 @@ class Driver:
         self.pos = np.zeros(w.n_sessions, dtype=np.int64)  # host copy of positions fed
         self.tdtype = torch.bfloat16 if w.dtype == "bf16" else torch.float32
         self.step_index = 0
+        self.stream = torch.cuda.current_stream().cuda_stream
         self.resident_out = torch.zeros(self.sizing["max_seq_per_call"], dtype=torch.int64,
                                         device=device)
 
@@ -130,7 +132,20 @@ class Driver:
             c.q = self._fill(V.TAG_Q, w.q_heads, tok_sess, tok_pos, w.q_scale)
             c.out = torch.empty((int(cu[-1]), w.q_heads, w.head_dim), dtype=self.tdtype,
                                 device=self.device)
+        self._bind(c)
         return c
+
+    def _bind(self, c: Call) -> None:
+        """Precompute the raw call arguments (done outside any timed region)."""
+        from paper_2609_31224_gb300._lib import host_i32
+        s_arr, s_p = host_i32(c.sessions)
+        c_arr, c_p = host_i32(c.cu)
+        q_ptrs = None
+        if c.q is not None:
+            base, stride = c.q.data_ptr(), c.q.stride(0) * c.q.element_size()
+            q_ptrs = [base + l * stride for l in range(self.w.layers)]
+        c.raw = (s_arr, s_p, c_arr, c_p, c.types.data_ptr(), c.k.data_ptr(), c.v.data_ptr(),
+                 q_ptrs, None if c.out is None else c.out.data_ptr())
 
     def prepare_step(self, with_q: bool = True) -> Step:
         """Generate (on the device) every input of the next step; advances host positions."""
@@ -161,16 +176,16 @@ class Driver:
                  on_append=None) -> int:
         """Append + (optionally) every layer's attention. Returns kernels launched."""
         cache = self.cache
-        cache.append_chunk(c.sessions, c.cu, c.types, c.k, c.v)
+        _, s_p, _, c_p, t_ptr, k_ptr, v_ptr, q_ptrs, o_ptr = c.raw
+        cache.append_chunk_raw(len(c.sessions), s_p, c_p, t_ptr, k_ptr, v_ptr, self.stream)
         if on_append is not None:
             on_append(c)
         launches = 2
         if attention and c.q is not None and c.kind != "prefix":
+            fn = cache.attn_prefill_raw if c.kind == "prefill" else cache.attn_decode_raw
+            stream = self.stream
             for layer in range(self.w.layers):
-                if c.kind == "prefill":
-                    cache.attn_prefill_chunk(layer, c.q[layer], c.out)
-                else:
-                    cache.attn_decode(layer, c.q[layer], c.out)
+                fn(layer, q_ptrs[layer], o_ptr, stream)
                 launches += 1
                 if on_attention is not None:
                     on_attention(c, layer)
