@@ -299,15 +299,25 @@ def run_e2e(drv, w, n_steps: int, world: int) -> dict:
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
+    # Inputs move on a copy stream, step by step in order; each step's compute waits
+    # only for its own inputs, so transfers of later steps overlap earlier compute.
+    copy_stream = torch.cuda.Stream()
+    ready = [torch.cuda.Event() for _ in steps]
     t0 = time.perf_counter()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    copy_stream.wait_stream(stream)
     h2d_total, d2h_total = 0, 0
+    with torch.cuda.stream(copy_stream):
+        for si in range(len(steps)):
+            for ci in range(len(steps[si].calls)):
+                for n, t in host[si][ci].items():
+                    dev[si][ci][n].copy_(t, non_blocking=True)
+                    h2d_total += t.numel() * t.element_size()
+            ready[si].record(copy_stream)
     for si, st in enumerate(steps):
+        stream.wait_event(ready[si])
         for ci, c in enumerate(st.calls):
-            for n, t in host[si][ci].items():
-                dev[si][ci][n].copy_(t, non_blocking=True)
-                h2d_total += t.numel() * t.element_size()
             drv.run_call(c)
             if c.out is not None:
                 out_host[si][ci].copy_(c.out, non_blocking=True)

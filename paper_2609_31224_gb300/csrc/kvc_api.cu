@@ -43,7 +43,8 @@ Sizes derive_sizes(const kvc_config& c) {
   const int64_t mv = (int64_t)c.max_seq_per_call * c.max_pages_per_session * PS;
   s.max_moves = (int)std::min<int64_t>(mv, 1 << 26);
   s.max_alloc = s.max_moves / PS + c.max_tokens_per_call / PS + 2 * c.max_seq_per_call + 1;
-  s.max_dec_items = (int)std::min<int64_t>(16384, std::max<int64_t>(256, (int64_t)c.max_seq_per_call * c.kv_heads * 32));
+  // Decode partial slots: two per CTA of the stream-K split (grid <= 2048 CTAs).
+  s.max_dec_items = 4096;
   s.max_pf_items = (int)std::min<int64_t>(2048, std::max<int64_t>(64, (int64_t)c.max_seq_per_call * c.kv_heads * 4));
   return s;
 }
@@ -162,7 +163,7 @@ struct kvc_ctx {
   int last_n_seq = 0, last_total = 0, last_max_t = 0;
   int attn_since_append = 0;  // attention launches since the last append
   bool last_single = false;
-  int dec_target = 0, pf_target = 0;
+  int pf_target = 0;
 };
 
 namespace {
@@ -268,7 +269,6 @@ int kvc_create(kvc_ctx** out, const kvc_config* cfg, void* d_pool, size_t pool_b
       launch_init(d, cfg->rope_base, s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess)
     return cleanup(fail(KVC_ECUDA, "initialisation failed: %s",
                         cudaGetErrorString(cudaGetLastError())));
-  ctx->dec_target = 4 * decode_grid_ctas(d);
   ctx->pf_target = 3 * prefill_grid_ctas(d);
   *out = ctx;
   return KVC_OK;
@@ -319,9 +319,9 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, const i
   AppendArgs a;
   a.n_seq = n_seq;
   a.total = total;
-  a.dec_target = ctx->dec_target;
+  a.dec_target = 0;  // decode uses the stream-K split
   a.pf_target = ctx->pf_target;
-  a.dec_min_blocks = 8;
+  a.dec_min_blocks = 0;
   a.pf_min_blocks = 4;
   for (int i = 0; i < n_seq; ++i) a.sessions[i] = h_sessions[i];
   for (int i = 0; i <= n_seq; ++i) a.cu[i] = h_cu_tokens[i];

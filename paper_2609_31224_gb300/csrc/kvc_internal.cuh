@@ -45,8 +45,8 @@ struct SeqInfo {
   int32_t live_head;
   int32_t n_live;
   int32_t n_blocks;     // n_hist_pages + n_live_pages
-  int32_t dec_chunks;   // split-K chunks of the decode work list
-  int32_t dec_base;     // first partial slot of this session (decode)
+  int32_t dec_chunks;   // unused by decode (stream-K split)
+  int32_t dec_base;     // first decode unit (session, kv head, page) of this session
   int32_t pf_chunks;
   int32_t pf_base;
   int32_t pad[3];
@@ -69,7 +69,8 @@ struct DevGlobals {
   int32_t n_pf_items;
   int32_t n_moves;
   int32_t total_tokens;
-  int32_t pad[8];
+  int32_t dec_nb_max;   // largest n_blocks among the last append's sessions
+  int32_t pad[7];
 };
 
 // Device pointers into the caller's workspace plus the shape, passed by value.

@@ -313,8 +313,19 @@ __global__ void __launch_bounds__(META_THREADS) append_plan_kernel(Dev d, Append
   }
   __syncthreads();
   // 4. Split-K work lists for decode and prefill attention.
-  build_worklist(d, n_seq, nb, a.dec_target, a.dec_min_blocks, d.max_dec_items, d.dec_items,
-                 true, s_warp, &s_total_dec);
+  // Decode splits the call's (session, kv head, page) units evenly over its CTAs
+  // (stream-K); it needs each session's first unit, the total and the largest session.
+  {
+    int total_units;
+    const int ubase = block_exclusive_scan(i < n_seq ? nb * d.kv_heads : 0, &total_units, s_warp);
+    const int nb_max = block_max(i < n_seq ? nb : 0, s_warp);
+    if (i < n_seq) d.seq[i].dec_base = ubase;
+    if (i == 0) {
+      s_total_dec = total_units;
+      d.g->dec_nb_max = nb_max;
+    }
+    __syncthreads();
+  }
   build_worklist(d, n_seq, nb, a.pf_target, a.pf_min_blocks, d.max_pf_items, d.pf_items, false,
                  s_warp, &s_total_pf);
   if (i == 0) {
