@@ -5,37 +5,34 @@
 // resident key (the compacted region, then the live region, the token's own
 // key included).
 //
-// Inside a CTA each of the 4 warps streams its own pages through a TMA
-// bulk-copy ring in shared memory, computes scores on CUDA cores (packed fp32
-// FMA), keeps a running max/sum with warp shuffles, and the CTA merges its
-// warps.  Two ways to spread the pages over CTAs (split-K):
+// Inside a CTA each warp streams its own pages through a TMA bulk-copy ring in
+// shared memory, computes scores on CUDA cores (packed fp32 FMA), keeps a
+// running max/sum with warp shuffles, and the CTA merges its warps.  Two ways
+// to spread the pages over CTAs (split-K):
 //   - stream-K (many sessions): the call's (session, head, page) units are cut
-//     into equal contiguous ranges, one per CTA; partial results go to global
-//     slots and the last CTA to arrive for a pair merges them (log-sum-exp);
-//   - clusters (few sessions): each (session, head) pair gets a cluster of
-//     CTAs that split its pages; the partial states are merged through
-//     distributed shared memory, with no global partials or atomics.
-#include <cooperative_groups.h>
-
+//     into equal contiguous ranges, one per CTA of 4 warps (three CTAs per SM);
+//   - pair split (few sessions): each (session, head) pair's pages are cut into
+//     k slices, one per CTA of 16 warps (one CTA per SM), so that every page of
+//     the call is in flight at once.
+// Either way partial states go to global slots and the last CTA to arrive for a
+// pair merges them (log-sum-exp).
 #include "kvc_internal.cuh"
-
-namespace cg = cooperative_groups;
 
 namespace kvc {
 
 namespace {
 
 constexpr unsigned FULL = 0xFFFFFFFFu;
-constexpr int DEC_WARPS = 4;
-constexpr int DEC_THREADS = DEC_WARPS * 32;
 constexpr int G = 4;  // query heads per KV head
-static_assert(DEC_WARPS == G, "the split-K merge maps one warp to one query row");
 constexpr float LOG2E = 1.4426950408889634f;
-constexpr int STAGES = 2;         // per-warp K/V ring depth
-constexpr int MAX_PARTS = 64;     // stream-K parts per (session, head), merge buffer size
+constexpr int MAX_PARTS = 64;     // partial states per (session, head) pair, at most
 
-template <typename T, int D>
+// One CTA shape: WARPS warps, each streaming its own pages through a STAGES-deep
+// ring of K/V tiles.
+template <typename T_, int D_, int WARPS_, int STAGES_>
 struct DecCfg {
+  using T = T_;
+  static constexpr int D = D_, WARPS = WARPS_, STAGES = STAGES_, THREADS = WARPS * 32;
   static constexpr int ESZ = sizeof(T);
   static constexpr int ROW_BYTES = D * ESZ;
   static_assert(ROW_BYTES == 256, "decode kernel assumes 256-byte K/V rows");
@@ -45,15 +42,25 @@ struct DecCfg {
   // shared memory per warp: STAGES x (K tile + V tile) + scores + probability
   // pairs (p, p) + alpha
   static constexpr int WARP_BYTES = STAGES * 2 * TILE + (G * PS + 2 * PS * G + G) * 4 + 16;
-  // The cross-warp merge (and the CTA result) reuse the stage buffers once every
-  // warp is done with its pages.
-  static constexpr int MERGE_FLOATS = DEC_WARPS * G * D + DEC_WARPS * G * 2;
-  static constexpr int RESULT_FLOATS = G * D + G * 2;
-  static_assert((MERGE_FLOATS + RESULT_FLOATS) * 4 <= DEC_WARPS * WARP_BYTES,
+  static_assert(WARP_BYTES % 16 == 0, "bulk-copy destinations must stay 16-byte aligned");
+  // The cross-warp merge reuses the stage buffers once every warp is done with
+  // its pages.
+  static constexpr int MERGE_FLOATS = WARPS * G * D + WARPS * G * 2;
+  static constexpr int RESULT_FLOATS = G * 2 + WARPS * G;
+  static_assert((MERGE_FLOATS + RESULT_FLOATS) * 4 <= WARPS * WARP_BYTES,
                 "merge area must fit in the stages");
-  static constexpr int SMEM = DEC_WARPS * WARP_BYTES + DEC_WARPS * STAGES * 8 +
-                              MAX_PARTS * G * 4 + 64;
+  static constexpr int SMEM = WARPS * WARP_BYTES + WARPS * STAGES * 8 + MAX_PARTS * G * 4 + 64;
 };
+
+// Stream-K kernel: 4 warps (one per query row in the split-K merge), 2-deep rings,
+// three CTAs per SM.
+template <typename T, int D>
+using SkCfg = DecCfg<T, D, 4, 2>;
+// Pair-split kernel: 16 warps, one tile pair each, one CTA per SM; with few
+// sessions every page of the call is in flight at once.
+constexpr int SP_WARPS = 16, SP_STAGES = 1;
+template <typename T, int D>
+using SpCfg = DecCfg<T, D, SP_WARPS, SP_STAGES>;
 
 template <typename T>
 __device__ inline void load_vec(const uint8_t* p, float* f);
@@ -83,41 +90,41 @@ __device__ inline void load_pv<float>(const uint8_t* p, float* f) {
 }
 
 // Shared-memory map of one CTA, as seen by one warp.
-template <typename T, int D>
+template <class C>
 struct Smem {
-  using C = DecCfg<T, D>;
   uint8_t* tiles;     // this warp's [STAGES][2][TILE]
   float* s_sc;        // [G][PS] scores
   float2* s_p2;       // [PS][G] probability pairs (p, p)
   float* s_alpha;     // [G]
   float* m_o;         // [W][G][D] warp partial outputs (aliases the stages)
   float* m_ml;        // [W][G][2]
-  float* r_o;         // [G][D] CTA result (aliases the stages)
-  float* r_ml;        // [G][2]
+  float* r_ml;        // [G][2] CTA (max, sum) per row
+  float* s_wsc;       // [W][G] weight of each warp's part (aliases the stages)
   uint64_t* wbars;    // this warp's [STAGES]
   float* s_scale;     // [MAX_PARTS][G]
   __device__ Smem(uint8_t* smem, int warp) {
     uint8_t* wbase = smem + warp * C::WARP_BYTES;
     tiles = wbase;
-    s_sc = reinterpret_cast<float*>(wbase + STAGES * 2 * C::TILE);
+    s_sc = reinterpret_cast<float*>(wbase + C::STAGES * 2 * C::TILE);
     s_p2 = reinterpret_cast<float2*>(s_sc + G * PS);
     s_alpha = reinterpret_cast<float*>(s_p2 + PS * G);
     m_o = reinterpret_cast<float*>(smem);
-    m_ml = m_o + DEC_WARPS * G * D;
-    r_o = m_ml + DEC_WARPS * G * 2;
-    r_ml = r_o + G * D;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + DEC_WARPS * C::WARP_BYTES);
-    wbars = bars + warp * STAGES;
-    s_scale = reinterpret_cast<float*>(bars + DEC_WARPS * STAGES);
+    m_ml = m_o + C::WARPS * G * C::D;
+    r_ml = m_ml + C::WARPS * G * 2;
+    s_wsc = r_ml + G * 2;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::WARPS * C::WARP_BYTES);
+    wbars = bars + warp * C::STAGES;
+    s_scale = reinterpret_cast<float*>(bars + C::WARPS * C::STAGES);
   }
 };
 
 // Blocks [blk_begin, blk_begin + nblk) of one (session, head) pair; warp w takes
-// blocks blk_begin + w, + w + 4, ...  Page ids are fetched 32 at a time (lane j
+// blocks blk_begin + w, + w + WARPS, ...  Page ids are fetched 32 at a time (lane j
 // holds the id of the warp's block win + j), so one round trip serves 32 loads.
-template <typename T, int D>
+template <class C>
 struct Segment {
-  using C = DecCfg<T, D>;
+  using T = typename C::T;
+  static constexpr int D = C::D;
   SeqInfo si;
   int head, blk_begin, nblk, n_my;
   const int32_t* hrow;
@@ -129,7 +136,7 @@ struct Segment {
     head = h;
     blk_begin = b0;
     nblk = nb;
-    n_my = (nblk > warp) ? (nblk - warp + DEC_WARPS - 1) / DEC_WARPS : 0;
+    n_my = (nblk > warp) ? (nblk - warp + C::WARPS - 1) / C::WARPS : 0;
     hrow = d.hist_pt + (size_t)si.sid * d.max_pages_per_session;
     lrow = d.live_pt + (size_t)si.sid * d.max_pages_per_session;
     pwin = -32;
@@ -137,17 +144,17 @@ struct Segment {
   }
 
   // Load the K and V tiles of this warp's k-th block (called by the whole warp).
-  __device__ void issue(const Dev& d, int layer, const Smem<T, D>& sm, uint32_t loads, int k,
+  __device__ void issue(const Dev& d, int layer, const Smem<C>& sm, uint32_t loads, int k,
                         int warp, int lane) {
     if (k >= pwin + 32) {
       pwin = k & ~31;
       const int j = pwin + lane;
-      pid = j < n_my ? block_page(si, hrow, lrow, blk_begin + warp + j * DEC_WARPS) : 0;
+      pid = j < n_my ? block_page(si, hrow, lrow, blk_begin + warp + j * C::WARPS) : 0;
     }
     const int page = __shfl_sync(FULL, pid, k - pwin);
     if (lane == 0) {
       const uint32_t n = loads + k;
-      const int st = n % STAGES;
+      const int st = n % C::STAGES;
       uint8_t* dst = sm.tiles + st * 2 * C::TILE;
       const T* kp = reinterpret_cast<const T*>(d.pool) +
                     pool_offset_elems(d, page, layer, 0, head, 0);
@@ -157,21 +164,22 @@ struct Segment {
     }
   }
 
-  __device__ void prefetch(const Dev& d, int layer, const Smem<T, D>& sm, uint32_t loads,
+  __device__ void prefetch(const Dev& d, int layer, const Smem<C>& sm, uint32_t loads,
                            int warp, int lane) {
     // The stage buffers may have been written by the previous merge.
     if (lane == 0) fence_proxy_async_smem();
-    for (int k = 0; k < min(STAGES, n_my); ++k) issue(d, layer, sm, loads, k, warp, lane);
+    for (int k = 0; k < min(C::STAGES, n_my); ++k) issue(d, layer, sm, loads, k, warp, lane);
   }
 };
 
 // Query rows of the G heads of `head`, rotated at the token's position and scaled
 // by log2(e)/sqrt(D).  Lane c holds 16-byte chunk c of each row; its rotate-half
 // partner is chunk c ^ 8.
-template <typename T, int D>
-__device__ void load_q(const Dev& d, const SeqInfo& si, int head, const T* q, float qk_scale,
-                       int lane, float (&qr)[G][DecCfg<T, D>::VEC]) {
-  using C = DecCfg<T, D>;
+template <class C>
+__device__ void load_q(const Dev& d, const SeqInfo& si, int head, const typename C::T* q,
+                       float qk_scale, int lane, float (&qr)[G][C::VEC]) {
+  using T = typename C::T;
+  constexpr int D = C::D;
   const int c = lane & 15;
   const uint8_t* qrow =
       reinterpret_cast<const uint8_t*>(q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G) * D);
@@ -195,20 +203,19 @@ __device__ void load_q(const Dev& d, const SeqInfo& si, int head, const T* q, fl
 // Stream this warp's blocks of the segment: scores, online softmax, P V.  The first
 // STAGES blocks must have been issued (Segment::prefetch).  Returns the first block
 // whose wait gave up, or -1.
-template <typename T, int D>
-__device__ int stream_pages(const Dev& d, int layer, Segment<T, D>& sg, const Smem<T, D>& sm,
-                            uint32_t loads, const float (&qr)[G][DecCfg<T, D>::VEC],
-                            float& m_run, float& l_run, float2 (&acc)[G][DecCfg<T, D>::PVD / 2],
-                            int warp, int lane) {
-  using C = DecCfg<T, D>;
+template <class C>
+__device__ int stream_pages(const Dev& d, int layer, Segment<C>& sg, const Smem<C>& sm,
+                            uint32_t loads, const float (&qr)[G][C::VEC], float& m_run,
+                            float& l_run, float2 (&acc)[G][C::PVD / 2], int warp, int lane) {
+  using T = typename C::T;
   const int half = lane >> 4, c = lane & 15;
   for (int k = 0; k < sg.n_my; ++k) {
     const uint32_t n = loads + k;
-    const int st = n % STAGES;
-    if (!__all_sync(FULL, mbar_wait(d, &sm.wbars[st], (n / STAGES) & 1))) return k;
+    const int st = n % C::STAGES;
+    if (!__all_sync(FULL, mbar_wait(d, &sm.wbars[st], (n / C::STAGES) & 1))) return k;
     const uint8_t* kt = sm.tiles + st * 2 * C::TILE;
     const uint8_t* vt = kt + C::TILE;
-    const BlockRange br = block_range(sg.si, sg.blk_begin + warp + k * DEC_WARPS);
+    const BlockRange br = block_range(sg.si, sg.blk_begin + warp + k * C::WARPS);
 
     // Scores: lanes 0-15 take even keys, 16-31 odd keys; each lane a 16-byte chunk.
 #pragma unroll
@@ -291,21 +298,20 @@ __device__ int stream_pages(const Dev& d, int layer, Segment<T, D>& sg, const Sm
       }
     }
     __syncwarp();
-    if (k + STAGES < sg.n_my) {
+    if (k + C::STAGES < sg.n_my) {
       if (lane == 0) fence_proxy_async_smem();
-      sg.issue(d, layer, sm, loads, k + STAGES, warp, lane);
+      sg.issue(d, layer, sm, loads, k + C::STAGES, warp, lane);
     }
   }
   return -1;
 }
 
 // After every warp of the CTA has finished (caller syncs): publish the warps'
-// partial states; after a second sync, merge_elem gives the CTA's (M, L, O) of
-// element e = g * D + dd.
-template <typename T, int D>
-__device__ void publish_warp(const Smem<T, D>& sm, float m_run, float l_run,
-                             const float2 (&acc)[G][DecCfg<T, D>::PVD / 2], int warp, int lane) {
-  using C = DecCfg<T, D>;
+// partial states.
+template <class C>
+__device__ void publish_warp(const Smem<C>& sm, float m_run, float l_run,
+                             const float2 (&acc)[G][C::PVD / 2], int warp, int lane) {
+  constexpr int D = C::D;
   if ((lane & 7) == 0) {
     sm.m_ml[(warp * G + (lane >> 3)) * 2 + 0] = m_run;
     sm.m_ml[(warp * G + (lane >> 3)) * 2 + 1] = l_run;
@@ -317,30 +323,167 @@ __device__ void publish_warp(const Smem<T, D>& sm, float m_run, float l_run,
       *reinterpret_cast<float2*>(&sm.m_o[(warp * G + g) * D + lane * C::PVD + 2 * j]) = acc[g][j];
 }
 
-template <typename T, int D>
-__device__ void merge_elem(const Smem<T, D>& sm, int e, float& M, float& L, float& O) {
-  const int g = e / D, dd = e % D;
-  float mw[DEC_WARPS];
-  M = -INFINITY;
+// After publish_warp and a sync: warp g < G reduces row g over the warps (max M,
+// sum L, each warp's weight exp2(m_w - M)); ends with a sync, after which
+// sm.r_ml holds (M, L) per row and merge_warps_elem(e) the row's unnormalised
+// output element e = g * D + dd.
+template <class C>
+__device__ void merge_warps(const Smem<C>& sm, int warp, int lane) {
+  static_assert(C::WARPS <= 32, "one lane per warp");
+  if (warp < G) {
+    const int g = warp;
+    float m = -INFINITY, l = 0.f;
+    if (lane < C::WARPS) {
+      const float2 ml = *reinterpret_cast<const float2*>(&sm.m_ml[(lane * G + g) * 2]);
+      m = ml.x;
+      l = ml.y;
+    }
+    float M = m;
 #pragma unroll
-  for (int w = 0; w < DEC_WARPS; ++w) {
-    mw[w] = sm.m_ml[(w * G + g) * 2];
-    M = fmaxf(M, mw[w]);
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(FULL, M, o));
+    const float w = exp2_safe(m, M);
+    float L = l * w;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(FULL, L, o);
+    if (lane < C::WARPS) sm.s_wsc[lane * G + g] = w;
+    if (lane == 0) {
+      sm.r_ml[g * 2 + 0] = M;
+      sm.r_ml[g * 2 + 1] = L;
+    }
   }
-  L = 0.f;
-  O = 0.f;
+  __syncthreads();
+}
+
+template <class C>
+__device__ inline float merge_warps_elem(const Smem<C>& sm, int e) {
+  constexpr int D = C::D;
+  const int g = e / D, dd = e % D;
+  float O = 0.f;
 #pragma unroll
-  for (int w = 0; w < DEC_WARPS; ++w) {
-    const float sc = exp2_safe(mw[w], M);
-    L += sm.m_ml[(w * G + g) * 2 + 1] * sc;
-    O += sm.m_o[(w * G + g) * D + dd] * sc;
+  for (int w = 0; w < C::WARPS; ++w) O += sm.m_o[(w * G + g) * D + dd] * sm.s_wsc[w * G + g];
+  return O;
+}
+
+// Arrive at a pair's counter after this CTA's partial state is written; true in
+// the last of `parts` CTAs to arrive.  One thread's acquire-release atomic after
+// the CTA barrier publishes every thread's partial writes and, in the last CTA,
+// orders the loads of the other parts after it.  Called by every thread.
+__device__ inline bool arrive_last(int* counter, int parts, int tid, int* s_flag) {
+  __syncthreads();
+  if (tid == 0) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;"
+                 : "=r"(old)
+                 : "l"(counter)
+                 : "memory");
+    *s_flag = old == parts - 1;
+  }
+  __syncthreads();
+  return *s_flag;
+}
+
+template <class C>
+__device__ inline void init_warp_barriers(uint64_t* wbars, int lane) {
+  if (lane == 0) {
+    for (int s = 0; s < C::STAGES; ++s) mbar_init(&wbars[s], 1);
+    fence_mbar_init();
   }
 }
 
-__device__ inline void init_warp_barriers(uint64_t* wbars, int lane) {
-  if (lane == 0) {
-    for (int s = 0; s < STAGES; ++s) mbar_init(&wbars[s], 1);
-    fence_mbar_init();
+// Warp-wide L2 prefetch of the query rows of `head` and the token's RoPE row, so
+// that load_q after pdl_wait() hits L2.
+template <class C>
+__device__ inline void prefetch_q(const Dev& d, const SeqInfo& si, int head,
+                                  const typename C::T* q, int lane) {
+  const uintptr_t qa =
+      reinterpret_cast<uintptr_t>(q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G) * C::D);
+  const uintptr_t ra = reinterpret_cast<uintptr_t>(d.rope + (size_t)si.pos_first * (C::D / 2));
+  const uintptr_t q0 = qa & ~uintptr_t(127), r0 = ra & ~uintptr_t(127);
+  const int nq = (int)((qa + G * C::ROW_BYTES - q0 + 127) / 128);  // <= 9 lines
+  const int nr = (int)((ra + C::D * 4 - r0 + 127) / 128);          // <= 5 lines
+  if (lane < nq) prefetch_l2(reinterpret_cast<const void*>(q0 + 128 * lane));
+  else if (lane >= 16 && lane - 16 < nr)
+    prefetch_l2(reinterpret_cast<const void*>(r0 + 128 * (lane - 16)));
+}
+
+// Log-sum-exp merge of the nch <= MAX_PARTS partial states of one (session, head)
+// pair into its G output rows (orow: row of query head head * G).  part(i) is the
+// slot holding part i.  Warp g < G reduces row g's maxima and sums from one pass
+// over the parts' (m, l) and leaves each part's weight, divided by the total, in
+// shared memory; then every thread sums its elements' weighted partial outputs
+// with up to 32 independent loads in flight.  Called by every thread of the CTA.
+template <class C, typename PartFn>
+__device__ void merge_parts(const Dev& d, const Smem<C>& sm, int nch, PartFn part,
+                            typename C::T* orow, int tid, int warp, int lane) {
+  using T = typename C::T;
+  constexpr int D = C::D;
+  static_assert(C::WARPS >= G, "one warp per query row");
+  constexpr int EPT = (G * D + C::THREADS - 1) / C::THREADS;  // elements per thread
+  constexpr int CH = 32 / EPT > 0 ? 32 / EPT : 1;              // parts per batch of loads
+  auto load_batch = [&](int c0, float (&a)[CH][EPT]) {
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      const bool ok = c0 + i < nch;
+      const float* b = d.dec_part_o + (size_t)(ok ? part(c0 + i) : 0) * G * D;
+#pragma unroll
+      for (int t = 0; t < EPT; ++t) {
+        const int e = tid + t * C::THREADS;
+        a[i][t] = (ok && e < G * D) ? __ldcg(b + e) : 0.f;
+      }
+    }
+  };
+  // The first batch of partial outputs is in flight while the weights are formed.
+  float a[CH][EPT];
+  load_batch(0, a);
+  if (warp < G) {
+    const int g = warp;
+    constexpr int PL = MAX_PARTS / 32;  // parts per lane
+    float2 ml[PL];
+    float M = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < PL; ++i) {
+      const int ch = lane + 32 * i;
+      ml[i] = ch < nch ? __ldcg(&d.dec_part_ml[(size_t)part(ch) * G + g])
+                       : make_float2(-INFINITY, 0.f);
+      M = fmaxf(M, ml[i].x);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(FULL, M, o));
+    float sc[PL], L = 0.f;
+#pragma unroll
+    for (int i = 0; i < PL; ++i) {
+      sc[i] = exp2_safe(ml[i].x, M);
+      L += ml[i].y * sc[i];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(FULL, L, o);
+    const float inv = 1.f / L;
+#pragma unroll
+    for (int i = 0; i < PL; ++i)
+      if (lane + 32 * i < nch) sm.s_scale[(lane + 32 * i) * G + g] = sc[i] * inv;
+  }
+  __syncthreads();
+  float O[EPT];
+#pragma unroll
+  for (int t = 0; t < EPT; ++t) O[t] = 0.f;
+  for (int c0 = 0;;) {
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      if (c0 + i >= nch) break;
+#pragma unroll
+      for (int t = 0; t < EPT; ++t) {
+        const int e = tid + t * C::THREADS;
+        if (e < G * D) O[t] += a[i][t] * sm.s_scale[(c0 + i) * G + e / D];
+      }
+    }
+    c0 += CH;
+    if (c0 >= nch) break;
+    load_batch(c0, a);
+  }
+#pragma unroll
+  for (int t = 0; t < EPT; ++t) {
+    const int e = tid + t * C::THREADS;
+    if (e < G * D) orow[e] = from_float<T>(O[t]);
   }
 }
 
@@ -348,16 +491,16 @@ __device__ inline void init_warp_barriers(uint64_t* wbars, int lane) {
 // Stream-K kernel.
 // ---------------------------------------------------------------------------
 template <typename T, int D>
-__global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int layer,
-                                                                  const T* __restrict__ q,
-                                                                  T* __restrict__ out,
-                                                                  float qk_scale, int min_units) {
-  using C = DecCfg<T, D>;
+__global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
+    Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale,
+    int min_units) {
+  using C = SkCfg<T, D>;
+  static_assert(C::WARPS == G, "the split-K merge maps one warp to one query row");
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const Smem<T, D> sm(smem, warp);
+  const Smem<C> sm(smem, warp);
   __shared__ int s_last, s_abort;
-  init_warp_barriers(sm.wbars, lane);
+  init_warp_barriers<C>(sm.wbars, lane);
   if (tid == 0) s_abort = 0;
   __syncthreads();
   // The next attention call may start its CTAs as soon as slots free up.  Before
@@ -399,32 +542,33 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
     const int pair_start = si.dec_base + head * nb, pair_end = pair_start + nb;
     const int seg_end = min(u_end, pair_end);
 
-    Segment<T, D> sg;
+    Segment<C> sg;
     sg.init(d, si, head, u - pair_start, seg_end - u, warp);
     sg.prefetch(d, layer, sm, loads, warp, lane);
     if (!waited) {
+      if (warp == 0) prefetch_q<C>(d, si, head, q, lane);
       pdl_wait();
       waited = true;
     }
     float qr[G][C::VEC];
-    load_q<T, D>(d, si, head, q, qk_scale, lane, qr);
+    load_q<C>(d, si, head, q, qk_scale, lane, qr);
     float m_run = -INFINITY, l_run = 0.f;  // for row lane >> 3
     float2 acc[G][C::PVD / 2];
 #pragma unroll
     for (int g = 0; g < G; ++g)
 #pragma unroll
       for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
-    const int failed_at = stream_pages<T, D>(d, layer, sg, sm, loads, qr, m_run, l_run, acc,
-                                             warp, lane);
+    const int failed_at = stream_pages<C>(d, layer, sg, sm, loads, qr, m_run, l_run, acc, warp,
+                                          lane);
     if (failed_at >= 0 && lane == 0) s_abort = 1;
     __syncthreads();
     if (s_abort) {
       // Some wait gave up: each warp drains the copies it still has in flight
       // (bounded waits), then the whole CTA stops together.
       if (failed_at >= 0) {
-        for (int k = failed_at; k < min(sg.n_my, failed_at + STAGES); ++k) {
+        for (int k = failed_at; k < min(sg.n_my, failed_at + C::STAGES); ++k) {
           const uint32_t n = loads + k;
-          mbar_wait(d, &sm.wbars[n % STAGES], (n / STAGES) & 1);
+          mbar_wait(d, &sm.wbars[n % C::STAGES], (n / C::STAGES) & 1);
         }
       }
       return;
@@ -432,95 +576,34 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
     loads += sg.n_my;
 
     // Merge the four warps' partial softmax states (stage buffers are free now).
-    publish_warp<T, D>(sm, m_run, l_run, acc, warp, lane);
+    publish_warp<C>(sm, m_run, l_run, acc, warp, lane);
     __syncthreads();
+    merge_warps<C>(sm, warp, lane);
     const bool whole = u == pair_start && seg_end == pair_end;
     const int slot = 2 * cta + (u == u_begin ? 0 : 1);
-    for (int e = tid; e < G * D; e += DEC_THREADS) {
-      float M, L, O;
-      merge_elem<T, D>(sm, e, M, L, O);
+    for (int e = tid; e < G * D; e += C::THREADS) {
+      const float O = merge_warps_elem<C>(sm, e);
       const int g = e / D, dd = e % D;
       if (whole) {
-        out[((size_t)si.q_row0 * d.q_heads + head * G + g) * D + dd] = from_float<T>(O / L);
+        out[((size_t)si.q_row0 * d.q_heads + head * G + g) * D + dd] =
+            from_float<T>(O / sm.r_ml[g * 2 + 1]);
       } else {
         d.dec_part_o[((size_t)slot * G + g) * D + dd] = O;
-        if (dd == 0) d.dec_part_ml[(size_t)slot * G + g] = make_float2(M, L);
+        if (dd == 0)
+          d.dec_part_ml[(size_t)slot * G + g] = make_float2(sm.r_ml[g * 2], sm.r_ml[g * 2 + 1]);
       }
     }
     if (!whole) {
       // The CTAs cf..cl own the pair's units; the last of them to arrive merges.
       const int cf = owner(pair_start), cl = owner(pair_end - 1);
       const int nch = cl - cf + 1;
-      __threadfence();
-      __syncthreads();
-      if (tid == 0) {
-        const int old = atomicAdd(&d.dec_count[seq * H + head], 1);
-        s_last = (old == nch - 1);
-      }
-      __syncthreads();
-      if (s_last) {
-        __threadfence();
+      if (arrive_last(&d.dec_count[seq * H + head], nch, tid, &s_last)) {
         // Slot of CTA cc's part of this pair: its first segment (2cc) unless the
         // pair began inside cf's range after its first unit (then 2cf+1).
         const int first_slot = start_of(cf) != pair_start ? 2 * cf + 1 : 2 * cf;
         auto slot_of = [&](int cc) { return cc == cf ? first_slot : 2 * cc; };
-        // Log-sum-exp merge: warp g reduces row g's maxima and sums over the parts,
-        // leaving each part's weight divided by the total in shared memory; then all
-        // threads sum the weighted partial outputs with independent loads in flight.
-        {
-          const int g = warp;  // DEC_WARPS == G
-          float M = -INFINITY;
-          for (int ch = lane; ch < nch; ch += 32)
-            M = fmaxf(M, __ldcg(&d.dec_part_ml[(size_t)slot_of(cf + ch) * G + g]).x);
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(FULL, M, o));
-          float L = 0.f;
-          for (int ch = lane; ch < nch; ch += 32) {
-            const float2 ml = __ldcg(&d.dec_part_ml[(size_t)slot_of(cf + ch) * G + g]);
-            const float sc = exp2_safe(ml.x, M);
-            sm.s_scale[ch * G + g] = sc;
-            L += ml.y * sc;
-          }
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(FULL, L, o);
-          const float inv = 1.f / L;
-          __syncwarp();
-          for (int ch = lane; ch < nch; ch += 32) sm.s_scale[ch * G + g] *= inv;
-        }
-        __syncthreads();
-        constexpr int EPT = G * D / DEC_THREADS;
-        float O[EPT];
-#pragma unroll
-        for (int i = 0; i < EPT; ++i) O[i] = 0.f;
-        // Eight parts per iteration: 8 x EPT independent loads in flight per thread.
-        int ch = 0;
-        for (; ch + 8 <= nch; ch += 8) {
-          float a[8][EPT];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const float* b = d.dec_part_o + (size_t)slot_of(cf + ch + k) * G * D;
-#pragma unroll
-            for (int i = 0; i < EPT; ++i) a[k][i] = __ldcg(b + tid + i * DEC_THREADS);
-          }
-#pragma unroll
-          for (int k = 0; k < 8; ++k)
-#pragma unroll
-            for (int i = 0; i < EPT; ++i)
-              O[i] += a[k][i] * sm.s_scale[(ch + k) * G + (tid + i * DEC_THREADS) / D];
-        }
-        for (; ch < nch; ++ch) {
-          const float* b0 = d.dec_part_o + (size_t)slot_of(cf + ch) * G * D;
-#pragma unroll
-          for (int i = 0; i < EPT; ++i) {
-            const int g = (tid + i * DEC_THREADS) / D;
-            O[i] += __ldcg(b0 + tid + i * DEC_THREADS) * sm.s_scale[ch * G + g];
-          }
-        }
-#pragma unroll
-        for (int i = 0; i < EPT; ++i) {
-          const int e = tid + i * DEC_THREADS;
-          out[((size_t)si.q_row0 * d.q_heads + head * G) * D + e] = from_float<T>(O[i]);
-        }
+        merge_parts<C>(d, sm, nch, [&](int ch) { return slot_of(cf + ch); },
+                       out + ((size_t)si.q_row0 * d.q_heads + head * G) * D, tid, warp, lane);
         if (tid == 0) d.dec_count[seq * H + head] = 0;
       }
     }
@@ -530,187 +613,131 @@ __global__ void __launch_bounds__(DEC_THREADS) attn_decode_kernel(Dev d, int lay
 }
 
 // ---------------------------------------------------------------------------
-// Cluster kernel: one cluster of CTAs per (session, head) pair; rank r takes
-// the r-th of `csize` equal slices of the pair's pages.  The CTA results are
-// merged by rank 0 through distributed shared memory.
+// Pair-split kernel (few sessions): CTA c takes slice c % k of pair c / k, the
+// pair's pages cut into k equal slices.  Each CTA's pages are issued before it
+// waits on the previous kernel; the k partial states of a pair are merged by
+// the last of its CTAs to finish.
 // ---------------------------------------------------------------------------
 template <typename T, int D>
-__global__ void __launch_bounds__(DEC_THREADS) attn_decode_cluster_kernel(
-    Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale) {
-  using C = DecCfg<T, D>;
+__global__ void __launch_bounds__(SpCfg<T, D>::THREADS, 1) attn_decode_split_kernel(
+    Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale, int k) {
+  using C = SpCfg<T, D>;
   extern __shared__ __align__(128) uint8_t smem[];
-  cg::cluster_group cluster = cg::this_cluster();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const Smem<T, D> sm(smem, warp);
-  const int rank = (int)cluster.block_rank(), csize = (int)cluster.num_blocks();
-  const int pair = blockIdx.x / csize;
-  const int H = d.kv_heads;
-  const int seq = pair / H, head = pair % H;
-  init_warp_barriers(sm.wbars, lane);
+  const Smem<C> sm(smem, warp);
+  __shared__ int s_last;
+  const int pair = blockIdx.x / k, slice = blockIdx.x % k;
+  const int seq = pair / d.kv_heads, head = pair % d.kv_heads;
+  init_warp_barriers<C>(sm.wbars, lane);
   __syncthreads();
   pdl_launch_dependents();
 
   const SeqInfo si = d.seq[seq];
   const int nb = si.n_blocks;
-  const int b0 = (int)((int64_t)rank * nb / csize), b1 = (int)((int64_t)(rank + 1) * nb / csize);
-  Segment<T, D> sg;
+  const int b0 = (int)((int64_t)slice * nb / k), b1 = (int)((int64_t)(slice + 1) * nb / k);
+  Segment<C> sg;
   sg.init(d, si, head, b0, b1 - b0, warp);
   sg.prefetch(d, layer, sm, 0, warp, lane);
+  if (warp == 0) prefetch_q<C>(d, si, head, q, lane);
   pdl_wait();
   float qr[G][C::VEC];
-  load_q<T, D>(d, si, head, q, qk_scale, lane, qr);
+  load_q<C>(d, si, head, q, qk_scale, lane, qr);
   float m_run = -INFINITY, l_run = 0.f;
   float2 acc[G][C::PVD / 2];
 #pragma unroll
   for (int g = 0; g < G; ++g)
 #pragma unroll
     for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
-  const int failed_at = stream_pages<T, D>(d, layer, sg, sm, 0, qr, m_run, l_run, acc, warp,
-                                           lane);
+  const int failed_at = stream_pages<C>(d, layer, sg, sm, 0, qr, m_run, l_run, acc, warp, lane);
   if (failed_at >= 0) {
     // A wait gave up (error recorded): drain this warp's copies, contribute nothing.
-    for (int k = failed_at; k < min(sg.n_my, failed_at + STAGES); ++k)
-      mbar_wait(d, &sm.wbars[k % STAGES], (k / STAGES) & 1);
+    for (int j = failed_at; j < min(sg.n_my, failed_at + C::STAGES); ++j)
+      mbar_wait(d, &sm.wbars[j % C::STAGES], (j / C::STAGES) & 1);
     m_run = -INFINITY;
     l_run = 0.f;
   }
   __syncthreads();
-  publish_warp<T, D>(sm, m_run, l_run, acc, warp, lane);
+  publish_warp<C>(sm, m_run, l_run, acc, warp, lane);
   __syncthreads();
-  for (int e = tid; e < G * D; e += DEC_THREADS) {
-    float M, L, O;
-    merge_elem<T, D>(sm, e, M, L, O);
-    sm.r_o[e] = O;
-    if ((e % D) == 0) {
-      sm.r_ml[(e / D) * 2 + 0] = M;
-      sm.r_ml[(e / D) * 2 + 1] = L;
+  merge_warps<C>(sm, warp, lane);
+  T* orow = out + ((size_t)si.q_row0 * d.q_heads + head * G) * D;
+  const int slot = blockIdx.x;
+  for (int e = tid; e < G * D; e += C::THREADS) {
+    const float O = merge_warps_elem<C>(sm, e);
+    const int g = e / D;
+    if (k == 1) {
+      orow[e] = from_float<T>(O / sm.r_ml[g * 2 + 1]);
+    } else {
+      d.dec_part_o[(size_t)slot * G * D + e] = O;
+      if ((e % D) == 0)
+        d.dec_part_ml[(size_t)slot * G + g] = make_float2(sm.r_ml[g * 2], sm.r_ml[g * 2 + 1]);
     }
   }
-  // Every rank's result is in its shared memory; rank 0 reads them all.  Every
-  // CTA reaches both cluster barriers (all earlier waits are bounded).
-  cluster.sync();
-  if (rank == 0) {
-    for (int e = tid; e < G * D; e += DEC_THREADS) {
-      const int g = e / D;
-      float M = -INFINITY;
-      for (int r = 0; r < csize; ++r) M = fmaxf(M, cluster.map_shared_rank(sm.r_ml, r)[g * 2]);
-      float L = 0.f, O = 0.f;
-      for (int r = 0; r < csize; ++r) {
-        const float* rml = cluster.map_shared_rank(sm.r_ml, r);
-        const float sc = exp2_safe(rml[g * 2], M);
-        L += rml[g * 2 + 1] * sc;
-        O += cluster.map_shared_rank(sm.r_o, r)[e] * sc;
-      }
-      out[((size_t)si.q_row0 * d.q_heads + head * G) * D + e] = from_float<T>(O / L);
-    }
-  }
-  // Keep this CTA's shared memory alive until rank 0 has read it.
-  cluster.sync();
+  if (k == 1) return;
+  if (!arrive_last(&d.dec_count[pair], k, tid, &s_last)) return;
+  merge_parts<C>(d, sm, k, [&](int ch) { return pair * k + ch; }, orow, tid, warp, lane);
+  if (tid == 0) d.dec_count[pair] = 0;
 }
 
+// Resident CTAs of the stream-K kernel (its grid), capped by the partial slots.
 template <typename T, int D>
-const void* dec_kernel_ptr() {
-  return reinterpret_cast<const void*>(&attn_decode_kernel<T, D>);
-}
-
-template <typename T, int D>
-int dec_smem() {
-  return DecCfg<T, D>::SMEM;
-}
-
-// Largest cluster size (16, else 8, else 0) with which the cluster kernel can run.
-template <typename T, int D>
-int cluster_size_for() {
-  const void* fn = reinterpret_cast<const void*>(&attn_decode_cluster_kernel<T, D>);
-  const int smem = dec_smem<T, D>();
-  if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
-    return 0;
-  cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  cudaGetLastError();
-  for (int cs : {16, 8}) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(cs);
-    cfg.blockDim = dim3(DEC_THREADS);
-    cfg.dynamicSmemBytes = smem;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = cs;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) == cudaSuccess && n > 0) return cs;
-    cudaGetLastError();
-  }
-  return 0;
-}
-
-template <typename T, int D>
-cudaError_t launch_cluster(const Dev& d, int layer, const T* q, T* out, float scale, int n_pairs,
-                           int cs, bool pdl, cudaStream_t s) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(n_pairs * cs);
-  cfg.blockDim = dim3(DEC_THREADS);
-  cfg.dynamicSmemBytes = dec_smem<T, D>();
-  cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = cs;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, &attn_decode_cluster_kernel<T, D>, d, layer, q, out, scale);
-}
-
-}  // namespace
-
-int decode_grid_ctas(const Dev& d) {
-  const void* fn = d.esz == 2 ? dec_kernel_ptr<__nv_bfloat16, 128>() : dec_kernel_ptr<float, 64>();
-  const int smem = d.esz == 2 ? dec_smem<__nv_bfloat16, 128>() : dec_smem<float, 64>();
+int stream_k_grid(const Dev& d) {
+  const void* fn = reinterpret_cast<const void*>(&attn_decode_kernel<T, D>);
+  const int smem = SkCfg<T, D>::SMEM;
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   int per_sm = 0;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, DEC_THREADS, smem);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SkCfg<T, D>::THREADS, smem);
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  return max(1, per_sm) * sms;
+  // Every CTA of the stream-K split may write two partial slots.
+  return min(d.max_dec_items / 2, max(1, per_sm) * sms);
+}
+
+// Resident CTAs of the pair-split kernel (one wave).
+template <typename T, int D>
+int split_slots() {
+  const void* fn = reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D>);
+  const int smem = SpCfg<T, D>::SMEM;
+  cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  int per_sm = 0;
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SpCfg<T, D>::THREADS, smem);
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return max(0, per_sm) * sms;
 }
 
 // Minimum (session, kv head, page) units per CTA of the stream-K split.
 constexpr int DEC_MIN_UNITS = 12;
+// The pair-split kernel takes calls whose pairs each get at least this many CTAs
+// in one wave.
+constexpr int SPLIT_MIN_K = 2;
+
+template <typename T, int D>
+cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int n_seq, bool pdl,
+                          cudaStream_t s) {
+  static thread_local const int grid = stream_k_grid<T, D>(d);
+  static thread_local const int slots = split_slots<T, D>();
+  const float scale = LOG2E / sqrtf((float)D);
+  const int n_pairs = n_seq * d.kv_heads;
+  const T* qt = static_cast<const T*>(q);
+  T* ot = static_cast<T*>(out);
+  const int k = n_pairs * SPLIT_MIN_K <= slots ? min(MAX_PARTS, slots / n_pairs) : 0;
+  if (k > 0)
+    return launch_ex(&attn_decode_split_kernel<T, D>, dim3(n_pairs * k),
+                     dim3(SpCfg<T, D>::THREADS), SpCfg<T, D>::SMEM, s, pdl, d, layer, qt, ot,
+                     scale, k);
+  return launch_ex(&attn_decode_kernel<T, D>, dim3(grid), dim3(SkCfg<T, D>::THREADS),
+                   SkCfg<T, D>::SMEM, s, pdl, d, layer, qt, ot, scale, DEC_MIN_UNITS);
+}
+
+}  // namespace
 
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                bool pdl, cudaStream_t s) {
-  static thread_local int grid_bf16 = 0, grid_f32 = 0, cs_bf16 = -1, cs_f32 = -1;
-  const float scale = LOG2E / sqrtf((float)d.head_dim);
-  // Every CTA of the stream-K split may write two partial slots.
-  const int max_grid = d.max_dec_items / 2;
-  const int n_pairs = n_seq * d.kv_heads;
-  if (d.esz == 2) {
-    if (!grid_bf16) grid_bf16 = min(max_grid, decode_grid_ctas(d));
-    if (cs_bf16 < 0) cs_bf16 = cluster_size_for<__nv_bfloat16, 128>();
-    // Few pairs: one cluster per pair, if the clusters fit in one wave.
-    if (cs_bf16 > 0 && n_pairs * cs_bf16 <= grid_bf16)
-      return launch_cluster<__nv_bfloat16, 128>(d, layer, static_cast<const __nv_bfloat16*>(q),
-                                                static_cast<__nv_bfloat16*>(out), scale, n_pairs,
-                                                cs_bf16, pdl, s);
-    return launch_ex(&attn_decode_kernel<__nv_bfloat16, 128>, dim3(grid_bf16), dim3(DEC_THREADS),
-                     dec_smem<__nv_bfloat16, 128>(), s, pdl, d, layer,
-                     static_cast<const __nv_bfloat16*>(q), static_cast<__nv_bfloat16*>(out), scale,
-                     DEC_MIN_UNITS);
-  }
-  if (!grid_f32) grid_f32 = min(max_grid, decode_grid_ctas(d));
-  if (cs_f32 < 0) cs_f32 = cluster_size_for<float, 64>();
-  if (cs_f32 > 0 && n_pairs * cs_f32 <= grid_f32)
-    return launch_cluster<float, 64>(d, layer, static_cast<const float*>(q),
-                                     static_cast<float*>(out), scale, n_pairs, cs_f32, pdl, s);
-  return launch_ex(&attn_decode_kernel<float, 64>, dim3(grid_f32), dim3(DEC_THREADS),
-                   dec_smem<float, 64>(), s, pdl, d, layer, static_cast<const float*>(q),
-                   static_cast<float*>(out), scale, DEC_MIN_UNITS);
+  if (d.esz == 2) return launch_decode<__nv_bfloat16, 128>(d, layer, q, out, n_seq, pdl, s);
+  return launch_decode<float, 64>(d, layer, q, out, n_seq, pdl, s);
 }
 
 }  // namespace kvc

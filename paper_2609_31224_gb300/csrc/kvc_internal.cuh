@@ -248,6 +248,13 @@ __device__ inline void pdl_launch_dependents() {
 }
 __device__ inline void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// Hint to bring the 128-byte line holding p into L2.  It has no effect on what
+// later loads observe (L2 is the coherence point), so it may run before
+// pdl_wait() on data the previous kernel is still writing.
+__device__ inline void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 // Launch with an optional programmatic-stream-serialization attribute.
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
@@ -324,7 +331,6 @@ cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out
                                bool pdl, cudaStream_t s);
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                 int max_t, bool pdl, cudaStream_t s);
-int decode_grid_ctas(const Dev& d);
 cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,
                                    const CUtensorMap& hi, const void* q, void* out, int grid,
                                    bool pdl, cudaStream_t s);
