@@ -173,18 +173,18 @@ struct Segment {
 };
 
 // Query rows of the G heads of `head`, rotated at the token's position and scaled
-// by log2(e)/sqrt(D).  Lane c holds 16-byte chunk c of each row; its rotate-half
-// partner is chunk c ^ 8.
+// by log2(e)/sqrt(D).  Lane c = lane & 7 holds 16-byte chunk c of each row
+// (qr[g][0, VEC)) and its rotate-half partner, chunk c + 8 (qr[g][VEC, 2 VEC)).
 template <class C>
 __device__ void load_q(const Dev& d, const SeqInfo& si, int head, const typename C::T* q,
-                       float qk_scale, int lane, float (&qr)[G][C::VEC]) {
+                       float qk_scale, int lane, float (&qr)[G][2 * C::VEC]) {
   using T = typename C::T;
   constexpr int D = C::D;
-  const int c = lane & 15;
+  static_assert(D / 2 * C::ESZ == 128, "rotate-half partner is chunk c + 8");
+  const int c = lane & 7;
   const uint8_t* qrow =
       reinterpret_cast<const uint8_t*>(q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G) * D);
-  const float2* cs = d.rope + (size_t)si.pos_first * (D / 2) + (c & 7) * C::VEC;
-  const bool lo = c < 8;
+  const float2* cs = d.rope + (size_t)si.pos_first * (D / 2) + c * C::VEC;
   float2 t[C::VEC];
 #pragma unroll
   for (int e = 0; e < C::VEC; ++e) t[e] = cs[e];
@@ -192,11 +192,12 @@ __device__ void load_q(const Dev& d, const SeqInfo& si, int head, const typename
   for (int g = 0; g < G; ++g) {
     float x[C::VEC], y[C::VEC];
     load_vec<T>(qrow + g * C::ROW_BYTES + c * 16, x);
-    load_vec<T>(qrow + g * C::ROW_BYTES + (c ^ 8) * 16, y);
+    load_vec<T>(qrow + g * C::ROW_BYTES + 128 + c * 16, y);
 #pragma unroll
-    for (int e = 0; e < C::VEC; ++e)
-      qr[g][e] = (lo ? fmaf(x[e], t[e].x, -y[e] * t[e].y) : fmaf(x[e], t[e].x, y[e] * t[e].y)) *
-                 qk_scale;
+    for (int e = 0; e < C::VEC; ++e) {
+      qr[g][e] = fmaf(x[e], t[e].x, -y[e] * t[e].y) * qk_scale;
+      qr[g][C::VEC + e] = fmaf(y[e], t[e].x, x[e] * t[e].y) * qk_scale;
+    }
   }
 }
 
@@ -205,10 +206,12 @@ __device__ void load_q(const Dev& d, const SeqInfo& si, int head, const typename
 // whose wait gave up, or -1.
 template <class C>
 __device__ int stream_pages(const Dev& d, int layer, Segment<C>& sg, const Smem<C>& sm,
-                            uint32_t loads, const float (&qr)[G][C::VEC], float& m_run,
+                            uint32_t loads, const float (&qr)[G][2 * C::VEC], float& m_run,
                             float& l_run, float2 (&acc)[G][C::PVD / 2], int warp, int lane) {
   using T = typename C::T;
-  const int half = lane >> 4, c = lane & 15;
+  const int kq = lane >> 3, c = lane & 7;
+  const bool up4 = lane & 4, up2 = lane & 2;
+  const int my_g = (up4 ? 2 : 0) + (up2 ? 1 : 0);  // row whose score this lane ends with
   for (int k = 0; k < sg.n_my; ++k) {
     const uint32_t n = loads + k;
     const int st = n % C::STAGES;
@@ -216,38 +219,39 @@ __device__ int stream_pages(const Dev& d, int layer, Segment<C>& sg, const Smem<
     const uint8_t* kt = sm.tiles + st * 2 * C::TILE;
     const uint8_t* vt = kt + C::TILE;
     const BlockRange br = block_range(sg.si, sg.blk_begin + warp + k * C::WARPS);
+    const bool interior = br.lo == 0 && br.hi == PS;
 
-    // Scores: lanes 0-15 take even keys, 16-31 odd keys; each lane a 16-byte chunk.
+    // Scores: the 8 lanes 8j..8j+7 take key 4i + j, lane c its chunks c and c + 8.
 #pragma unroll
-    for (int i = 0; i < PS / 2; ++i) {
-      const int key = 2 * i + half;
-      float kf[C::VEC];
-      load_vec<T>(kt + key * C::ROW_BYTES + c * 16, kf);
+    for (int i = 0; i < PS / 4; ++i) {
+      const int key = 4 * i + kq;
+      float k0[C::VEC], k1[C::VEC];
+      load_vec<T>(kt + key * C::ROW_BYTES + c * 16, k0);
+      load_vec<T>(kt + key * C::ROW_BYTES + 128 + c * 16, k1);
       float a[G];
 #pragma unroll
       for (int g = 0; g < G; ++g) {
         // Even and odd dims accumulate in the two halves of a packed pair.
         float2 acc2 = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int e = 0; e < C::VEC; e += 2)
-          acc2 = __ffma2_rn(make_float2(qr[g][e], qr[g][e + 1]), make_float2(kf[e], kf[e + 1]),
+        for (int e = 0; e < C::VEC; e += 2) {
+          acc2 = __ffma2_rn(make_float2(qr[g][e], qr[g][e + 1]), make_float2(k0[e], k0[e + 1]),
                             acc2);
+          acc2 = __ffma2_rn(make_float2(qr[g][C::VEC + e], qr[g][C::VEC + e + 1]),
+                            make_float2(k1[e], k1[e + 1]), acc2);
+        }
         a[g] = acc2.x + acc2.y;
       }
-      // Reduce-scatter of 4 sums over 16 lanes, then all-reduce over 4.
-      const bool up8 = lane & 8;
-      const float r0 = __shfl_xor_sync(FULL, up8 ? a[0] : a[2], 8);
-      const float r1 = __shfl_xor_sync(FULL, up8 ? a[1] : a[3], 8);
-      const float b0 = (up8 ? a[2] : a[0]) + r0;
-      const float b1 = (up8 ? a[3] : a[1]) + r1;
-      const bool up4 = lane & 4;
-      float v = (up4 ? b1 : b0) + __shfl_xor_sync(FULL, up4 ? b0 : b1, 4);
-      v += __shfl_xor_sync(FULL, v, 2);
+      // Reduce-scatter of the 4 sums over the key's 8 lanes (xor 4, then xor 2),
+      // then a pair sum (xor 1): lane ends with row my_g's score.
+      const float r0 = __shfl_xor_sync(FULL, up4 ? a[0] : a[2], 4);
+      const float r1 = __shfl_xor_sync(FULL, up4 ? a[1] : a[3], 4);
+      const float b0 = (up4 ? a[2] : a[0]) + r0;
+      const float b1 = (up4 ? a[3] : a[1]) + r1;
+      float v = (up2 ? b1 : b0) + __shfl_xor_sync(FULL, up2 ? b0 : b1, 2);
       v += __shfl_xor_sync(FULL, v, 1);
-      if ((lane & 3) == 0) {
-        const int g = (up8 ? 2 : 0) + (up4 ? 1 : 0);
-        sm.s_sc[g * PS + key] = (key >= br.lo && key < br.hi) ? v : -INFINITY;
-      }
+      if ((lane & 1) == 0)
+        sm.s_sc[my_g * PS + key] = (interior || (key >= br.lo && key < br.hi)) ? v : -INFINITY;
     }
     __syncwarp();
     // Online softmax: lane handles row lane>>3, keys 2*(lane&7) and +1.
@@ -275,12 +279,15 @@ __device__ int stream_pages(const Dev& d, int layer, Segment<C>& sg, const Smem<
     // PV: lane owns dims [PVD*lane, PVD*lane + PVD) of all G rows, as packed pairs.
     {
       const float4 al = *reinterpret_cast<const float4*>(sm.s_alpha);
-      const float alv[G] = {al.x, al.y, al.z, al.w};
+      // Rescale only when some row's running max moved (warp-uniform).
+      if (al.x != 1.f || al.y != 1.f || al.z != 1.f || al.w != 1.f) {
+        const float alv[G] = {al.x, al.y, al.z, al.w};
 #pragma unroll
-      for (int g = 0; g < G; ++g)
+        for (int g = 0; g < G; ++g)
 #pragma unroll
-        for (int j = 0; j < C::PVD / 2; ++j)
-          acc[g][j] = __fmul2_rn(acc[g][j], make_float2(alv[g], alv[g]));
+          for (int j = 0; j < C::PVD / 2; ++j)
+            acc[g][j] = __fmul2_rn(acc[g][j], make_float2(alv[g], alv[g]));
+      }
 #pragma unroll
       for (int key = 0; key < PS; ++key) {
         const float4 p01 = *reinterpret_cast<const float4*>(sm.s_p2 + key * G);
@@ -550,7 +557,7 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
       pdl_wait();
       waited = true;
     }
-    float qr[G][C::VEC];
+    float qr[G][2 * C::VEC];
     load_q<C>(d, si, head, q, qk_scale, lane, qr);
     float m_run = -INFINITY, l_run = 0.f;  // for row lane >> 3
     float2 acc[G][C::PVD / 2];
@@ -640,7 +647,7 @@ __global__ void __launch_bounds__(SpCfg<T, D>::THREADS, 1) attn_decode_split_ker
   sg.prefetch(d, layer, sm, 0, warp, lane);
   if (warp == 0) prefetch_q<C>(d, si, head, q, lane);
   pdl_wait();
-  float qr[G][C::VEC];
+  float qr[G][2 * C::VEC];
   load_q<C>(d, si, head, q, qk_scale, lane, qr);
   float m_run = -INFINITY, l_run = 0.f;
   float2 acc[G][C::PVD / 2];
