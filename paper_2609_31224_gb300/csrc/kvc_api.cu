@@ -45,7 +45,9 @@ Sizes derive_sizes(const kvc_config& c) {
   s.max_alloc = s.max_moves / PS + c.max_tokens_per_call / PS + 2 * c.max_seq_per_call + 1;
   // Decode partial slots: two per CTA of the stream-K split (grid <= 2048 CTAs).
   s.max_dec_items = 4096;
-  s.max_pf_items = (int)std::min<int64_t>(2048, std::max<int64_t>(64, (int64_t)c.max_seq_per_call * c.kv_heads * 4));
+  // Prefill partial slots: the binary32 kernel's chunk list, and two per CTA of the
+  // bfloat16 kernel's stream-K split.
+  s.max_pf_items = (int)std::min<int64_t>(2048, std::max<int64_t>(512, (int64_t)c.max_seq_per_call * c.kv_heads * 4));
   return s;
 }
 

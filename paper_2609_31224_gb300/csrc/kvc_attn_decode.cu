@@ -377,14 +377,7 @@ __device__ inline float merge_warps_elem(const Smem<C>& sm, int e) {
 // orders the loads of the other parts after it.  Called by every thread.
 __device__ inline bool arrive_last(int* counter, int parts, int tid, int* s_flag) {
   __syncthreads();
-  if (tid == 0) {
-    int old;
-    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;"
-                 : "=r"(old)
-                 : "l"(counter)
-                 : "memory");
-    *s_flag = old == parts - 1;
-  }
+  if (tid == 0) *s_flag = arrive_acq_rel(counter, parts);
   __syncthreads();
   return *s_flag;
 }
@@ -516,38 +509,19 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
   pdl_launch_dependents();
   bool waited = false;
 
-  // The call's (session, KV head, page) units, session-major, are cut into n_cta
-  // equal contiguous ranges, one per CTA.  A range covers "segments" (the part of
-  // one (session, head) pair inside it); only its first and last segments can be
-  // partial, and they go to partial slots 2c and 2c+1.
+  // Stream-K: this CTA's contiguous range of the call's units (UnitSplit).
   const int H = d.kv_heads;
-  const int U = d.g->n_dec_items;  // units of this call
-  const int n_seq = d.g->n_seq;
-  // n_cta: at most the grid, at least min_units units per CTA, and small enough that
-  // no (session, head) pair spans more than MAX_PARTS CTAs (the merge's buffer).
-  const int nb_max = max(1, d.g->dec_nb_max);
-  const int c_parts = (int)((int64_t)U * (MAX_PARTS - 2) / (nb_max + MAX_PARTS - 2));
-  const int n_cta = max(1, min((int)gridDim.x, min((U + min_units - 1) / min_units, c_parts)));
-  if ((int)blockIdx.x >= n_cta) return;
+  const UnitSplit us = unit_split(d, gridDim.x, min_units, MAX_PARTS);
+  if ((int)blockIdx.x >= us.n_cta) return;
   const int cta = blockIdx.x;
-  auto start_of = [&](int cc) { return (int)((int64_t)cc * U / n_cta); };
-  auto owner = [&](int64_t u) { return (int)(((u + 1) * n_cta - 1) / U); };
-  const int u_begin = start_of(cta), u_end = start_of(cta + 1);
+  const int u_begin = us.start_of(cta), u_end = us.start_of(cta + 1);
   uint32_t loads = 0;  // loads issued (== consumed) by this warp so far
 
   for (int u = u_begin; u < u_end;) {
-    // Session of unit u: the last one whose first unit is <= u.
-    int lo = 0, hi = n_seq - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (d.seq[mid].dec_base <= u) lo = mid; else hi = mid - 1;
-    }
-    const int seq = lo;
-    const SeqInfo si = d.seq[seq];
-    const int nb = si.n_blocks;
-    const int head = (u - si.dec_base) / nb;
-    const int pair_start = si.dec_base + head * nb, pair_end = pair_start + nb;
-    const int seg_end = min(u_end, pair_end);
+    const UnitSeg seg = unit_segment(d, u, u_end);
+    const SeqInfo& si = seg.si;
+    const int seq = seg.seq, head = seg.head;
+    const int pair_start = seg.pair_start, pair_end = seg.pair_end, seg_end = seg.end;
 
     Segment<C> sg;
     sg.init(d, si, head, u - pair_start, seg_end - u, warp);
@@ -602,14 +576,11 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
     }
     if (!whole) {
       // The CTAs cf..cl own the pair's units; the last of them to arrive merges.
-      const int cf = owner(pair_start), cl = owner(pair_end - 1);
+      const int cf = us.owner(pair_start), cl = us.owner(pair_end - 1);
       const int nch = cl - cf + 1;
       if (arrive_last(&d.dec_count[seq * H + head], nch, tid, &s_last)) {
-        // Slot of CTA cc's part of this pair: its first segment (2cc) unless the
-        // pair began inside cf's range after its first unit (then 2cf+1).
-        const int first_slot = start_of(cf) != pair_start ? 2 * cf + 1 : 2 * cf;
-        auto slot_of = [&](int cc) { return cc == cf ? first_slot : 2 * cc; };
-        merge_parts<C>(d, sm, nch, [&](int ch) { return slot_of(cf + ch); },
+        const int first_slot = us.slot_of(cf, cf, pair_start);
+        merge_parts<C>(d, sm, nch, [&](int ch) { return ch ? 2 * (cf + ch) : first_slot; },
                        out + ((size_t)si.q_row0 * d.q_heads + head * G) * D, tid, warp, lane);
         if (tid == 0) d.dec_count[seq * H + head] = 0;
       }

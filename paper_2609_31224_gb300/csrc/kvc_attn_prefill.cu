@@ -10,6 +10,8 @@
 // CUDA-core kernel (one thread per query row).
 #include <cuda.h>
 
+#include <algorithm>
+
 #include "kvc_internal.cuh"
 
 namespace kvc {
@@ -251,7 +253,9 @@ cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* ou
       if (!make_pool_maps(d, maps)) return cudaErrorInvalidValue;
     }
     if (!gtc) gtc = pf_grid<0>(prefill_tc_kernel_ptr(), prefill_tc_threads(), prefill_tc_smem());
-    return launch_attn_prefill_tc(d, layer, maps.lo, maps.hi, q, out, gtc, pdl, s);
+    // Each CTA of the stream-K split may write two partial slots.
+    return launch_attn_prefill_tc(d, layer, maps.lo, maps.hi, q, out,
+                                  std::min(gtc, d.max_pf_items / 2), pdl, s);
   }
   const float scale = LOG2E / sqrtf((float)d.head_dim);
   static thread_local int gf = 0;

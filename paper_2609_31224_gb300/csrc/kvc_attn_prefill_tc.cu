@@ -1,15 +1,20 @@
 // Chunked-prefill GQA attention on the 5th-generation tensor cores (tcgen05 +
 // TMEM), bfloat16 K/V/q, fp32 softmax and accumulation.
 //
-// Per work item (session, KV head, chunk of resident pages) the T*G query rows
-// (T <= 32 tokens, G = 4 heads) form the M = 128 rows of an MMA tile; the
-// rows past T*G are zero padding.  Warp roles in one CTA:
-//   warp 0    producer: 2-D TMA loads (128-byte swizzle) of 4 K/V pages
-//             (64 keys) per stage into a shared-memory ring;
-//   warp 1    MMA issuer: one elected thread issues tcgen05.mma from
-//             shared-memory descriptors, S = Q K^T (N = 64) into a
-//             double-buffered TMEM tile and O += P V (N = 128) into TMEM;
-//             completion is signalled with tcgen05.commit on mbarriers;
+// The call's (session, KV head, page) units are cut into equal contiguous
+// ranges, one per CTA (stream-K); per segment (the part of one (session, KV
+// head) pair in a range) the T*G query rows (T <= 32 tokens, G = 4 heads) form
+// the M = 128 rows of an MMA tile, the rows past T*G being zero padding.  A
+// pair split over several CTAs is merged by the last of them (log-sum-exp).
+// Warp roles in one CTA:
+//   warps 0, 6 producers: 2-D TMA loads (128-byte swizzle) of the K (warp 0)
+//             and V (warp 6) tiles of 4 pages (64 keys) per stage into a
+//             shared-memory ring whose K and V halves are released separately;
+//   warps 1, 7 MMA issuers: one elected thread each issues tcgen05.mma, warp
+//             1 S = Q K^T (N = 64, Q from TMEM, K from shared memory) into a
+//             double-buffered TMEM tile, warp 7 O += P V (N = 128, P from
+//             TMEM, V from shared memory) into TMEM; completion is signalled
+//             with tcgen05.commit on mbarriers;
 //   warps 2-5 softmax: each thread owns one TMEM lane (= one query row):
 //             it builds its rotated, scaled query row in shared memory,
 //             reads its row of S from TMEM, masks (resident slots, causal
@@ -29,38 +34,46 @@ constexpr int G = 4;
 constexpr int D = 128;
 constexpr int M = 128;                       // MMA rows (query rows, padded)
 constexpr int NK = 64;                       // keys per stage (4 pages)
-constexpr int TC_STAGES = 4;                 // K/V stages
+constexpr int TC_STAGES = 7;                 // K/V stages: all of shared memory
 constexpr int KV_PANEL = NK * 128;           // 64 rows x 128 B = 8 KiB
 constexpr int STAGE = 4 * KV_PANEL;          // K lo, K hi, V lo, V hi = 32 KiB
-constexpr int Q_PANEL = M * 128;             // 16 KiB
-constexpr int Q_BYTES = 2 * Q_PANEL;         // 32 KiB
-constexpr int P_BYTES = M * 128;             // 128 rows x 64 keys bf16 = 16 KiB
-constexpr int TMEM_COLS = 256;               // S0 [0,64) S1 [64,128) O [128,256)
-constexpr int S_COL = 0, O_COL = 128;
+// Tensor memory (512 columns x 128 lanes of 32 bits; lane = query row):
+//   S0 [0,64) S1 [64,128)  fp32 scores of two stages
+//   O  [128,256)           fp32 output accumulator
+//   P0 [256,288) P1 [288,320)  bfloat16 probabilities (2 per column), MMA A operand
+//   Q  [320,384)           bfloat16 rotated, scaled query rows, MMA A operand
+constexpr int TMEM_COLS = 512;
+constexpr int S_COL = 0, O_COL = 128, P_COL = 256, Q_COL = 320;
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr float RESCALE_LOG2 = 8.f;          // rescale O only when the max grows by > 2^8
-constexpr int THREADS = 6 * 32;
+constexpr int THREADS = 8 * 32;
+constexpr int PF_MIN_UNITS = 16;              // pages per CTA of the stream-K split, at least
+constexpr int PF_MAX_PARTS = 1 << 16;        // no limit on CTAs per pair (merged row by row)
 constexpr unsigned FULL = 0xFFFFFFFFu;
 
-// Shared memory map (offsets from a 1024-aligned base).
-constexpr int OFF_Q = 0;
-constexpr int OFF_KV = OFF_Q + Q_BYTES;
-constexpr int OFF_P = OFF_KV + TC_STAGES * STAGE;
-constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+// Shared memory map (offsets from a 1024-aligned base): the K/V ring, barriers.
+constexpr int OFF_KV = 0;
+constexpr int OFF_BAR = OFF_KV + TC_STAGES * STAGE;
 enum {
-  B_KV_FULL = 0,                         // [TC_STAGES]
-  B_KV_EMPTY = B_KV_FULL + TC_STAGES,    // [TC_STAGES]
-  B_S_FULL = B_KV_EMPTY + TC_STAGES,     // [2]
+  B_K_FULL = 0,                          // [TC_STAGES] K half of a stage loaded
+  B_K_EMPTY = B_K_FULL + TC_STAGES,      // [TC_STAGES] ... and read by S = Q K^T
+  B_V_FULL = B_K_EMPTY + TC_STAGES,      // [TC_STAGES] V half loaded
+  B_V_EMPTY = B_V_FULL + TC_STAGES,      // [TC_STAGES] ... and read by O += P V
+  B_S_FULL = B_V_EMPTY + TC_STAGES,      // [2]
   B_S_EMPTY = B_S_FULL + 2,              // [2]
   B_P_FULL = B_S_EMPTY + 2,              // [2]
   B_P_EMPTY = B_P_FULL + 2,              // [2]
-  B_O = B_P_EMPTY + 2,                   // one phase per P V product
-  B_Q = B_O + 1,                         // one phase per item (query tile ready)
-  B_FINAL = B_Q + 1,                     // every MMA of the CTA complete
+  // [2] P V product j complete: barrier j % 2, phase j / 2.  One barrier per P
+  // buffer keeps every waiter at most one phase behind (P V products j - 3 and
+  // earlier are known complete when j is waited for), so parity waits are exact.
+  B_O = B_P_EMPTY + 2,
+  B_Q = B_O + 2,                         // one phase per segment (query tile ready)
+  B_FINAL = B_Q + 1,                     // every MMA of the CTA complete (both issuers)
   N_BARS = B_FINAL + 1
 };
 constexpr int OFF_TMEM_ADDR = OFF_BAR + N_BARS * 8;
 constexpr int TC_SMEM = OFF_TMEM_ADDR + 16 + 1024;  // + alignment slack
+static_assert(TC_SMEM <= 227 * 1024, "shared memory per CTA");
 
 // -- tcgen05 helpers ------------------------------------------------------------------
 __device__ inline void tmem_alloc(uint32_t* smem_dst, uint32_t ncols) {
@@ -86,13 +99,15 @@ __device__ inline void tc_commit(uint64_t* bar) {
           smem_u32(bar))
       : "memory");
 }
-__device__ inline void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                              uint32_t accumulate) {
+// D (TMEM) (+)= A B with A read from tensor memory (M lanes, K/2 columns of
+// bfloat16 pairs) and B from shared memory.
+__device__ inline void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                 uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 // Each thread of the warp reads 32 consecutive fp32 columns of its TMEM lane.
@@ -111,6 +126,19 @@ __device__ inline void tmem_ld32(uint32_t taddr, float* v) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ inline void tmem_st32(uint32_t taddr, const uint32_t* w) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+      "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
+          taddr),
+      "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7]),
+      "r"(w[8]), "r"(w[9]), "r"(w[10]), "r"(w[11]), "r"(w[12]), "r"(w[13]), "r"(w[14]),
+      "r"(w[15]), "r"(w[16]), "r"(w[17]), "r"(w[18]), "r"(w[19]), "r"(w[20]), "r"(w[21]),
+      "r"(w[22]), "r"(w[23]), "r"(w[24]), "r"(w[25]), "r"(w[26]), "r"(w[27]), "r"(w[28]),
+      "r"(w[29]), "r"(w[30]), "r"(w[31])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 __device__ inline void tmem_st32(uint32_t taddr, const float* v) {
   asm volatile(
@@ -171,18 +199,6 @@ __device__ inline float ex2(float x) {
   return y;
 }
 
-// 16-byte chunk `c` (0..7) of row `r` of a 128-byte-swizzled panel.
-__device__ inline uint32_t sw128(uint32_t panel, int r, int c) {
-  return panel + r * 128 + ((c ^ (r & 7)) << 4);
-}
-
-__device__ inline void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
-                                    uint32_t e) {
-  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
-               "r"(e)
-               : "memory");
-}
-
 __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
     Dev d, int layer, const __grid_constant__ CUtensorMap map_lo,
     const __grid_constant__ CUtensorMap map_hi, const __nv_bfloat16* __restrict__ q,
@@ -198,8 +214,10 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
 
   if (tid == 0) {
     for (int s = 0; s < TC_STAGES; ++s) {
-      mbar_init(&bars[B_KV_FULL + s], 1);
-      mbar_init(&bars[B_KV_EMPTY + s], 1);
+      mbar_init(&bars[B_K_FULL + s], 1);
+      mbar_init(&bars[B_K_EMPTY + s], 1);
+      mbar_init(&bars[B_V_FULL + s], 1);
+      mbar_init(&bars[B_V_EMPTY + s], 1);
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&bars[B_S_FULL + s], 1);
@@ -207,15 +225,15 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       mbar_init(&bars[B_P_FULL + s], 4);
       mbar_init(&bars[B_P_EMPTY + s], 1);
     }
-    mbar_init(&bars[B_O], 1);
+    mbar_init(&bars[B_O + 0], 1);
+    mbar_init(&bars[B_O + 1], 1);
     mbar_init(&bars[B_Q], 4);
-    mbar_init(&bars[B_FINAL], 1);
+    mbar_init(&bars[B_FINAL], 2);
     fence_mbar_init();
     s_abort = 0;
   }
-  // Zero the query, K/V and P tiles once: padding query rows stay zero, and the
-  // keys of partly filled stages only ever hold finite values (their weights are
-  // 0, and 0 times a stale NaN would not be 0).
+  // Zero the K/V ring once: the keys of partly filled stages only ever hold finite
+  // values (their weights are 0, and 0 times a stale NaN would not be 0).
   for (int i = tid; i < OFF_BAR / 16; i += THREADS)
     reinterpret_cast<uint4*>(smem)[i] = make_uint4(0, 0, 0, 0);
   fence_proxy_async_smem();
@@ -229,36 +247,45 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
   pdl_launch_dependents();
 
   const int H = d.kv_heads, L = d.layers;
-  const int n_items = d.g->n_pf_items * H;
-  const uint32_t sQ = smem_u32(smem + OFF_Q);
+  // Stream-K: this CTA's contiguous range of the call's units (UnitSplit); the three
+  // roles walk the same segments of it.
+  const UnitSplit us = unit_split(d, gridDim.x, PF_MIN_UNITS, PF_MAX_PARTS);
+  const int cta = blockIdx.x;
+  const bool active = cta < us.n_cta;
+  const int u_begin = active ? us.start_of(cta) : 0, u_end = active ? us.start_of(cta + 1) : 0;
   const uint32_t sKV = smem_u32(smem + OFF_KV);
-  const uint32_t sP = smem_u32(smem + OFF_P);
 
-  if (warp == 0) {
-    // ---------------- producer ----------------
-    // The whole warp walks the items; lane j fetches the page id of block
-    // (window + j) so that one round trip serves 32 blocks, and lane 0 issues the
-    // TMA loads with the ids shuffled to it.
+  if (warp == 0 || warp == 6) {
+    // ---------------- producers ----------------
+    // Warp 0 loads the K halves of the stages, warp 6 the V halves, each with its
+    // own full/empty barriers: a K half is free again once S = Q K^T of its stage
+    // is complete, a V half once O += P V is, so the K loads run ahead of the V
+    // loads by up to the ring depth.  The whole warp walks the segments; lane j
+    // fetches the page id of block (window + j) so that one round trip serves 32
+    // blocks, and lane 0 issues the TMA loads with the ids shuffled to it.
+    const bool is_v = warp == 6;
+    const int b_full = is_v ? B_V_FULL : B_K_FULL, b_empty = is_v ? B_V_EMPTY : B_K_EMPTY;
     uint32_t n = 0;  // stages produced
     bool stop = false;
-    for (int it = blockIdx.x; it < n_items && !stop; it += gridDim.x) {
-      const int item = it / H, head = it % H;
-      const Item itm = d.pf_items[item];
-      const SeqInfo si = d.seq[itm.seq];
+    for (int u = u_begin; u < u_end && !stop;) {
+      const UnitSeg seg = unit_segment(d, u, u_end);
+      u = seg.end;
+      const int head = seg.head;
+      const SeqInfo& si = seg.si;
       const int32_t* hrow = d.hist_pt + (size_t)si.sid * d.max_pages_per_session;
       const int32_t* lrow = d.live_pt + (size_t)si.sid * d.max_pages_per_session;
-      const int nblk = itm.blk_end - itm.blk_begin;
+      const int blk0 = seg.blk_begin(), nblk = seg.end - seg.u;
       const int n_st = (nblk + 3) / 4;
       int pid = 0;
       for (int k = 0; k < n_st; ++k, ++n) {
         const int b0 = 4 * k;
         if ((b0 & 31) == 0) {
           const int bj = b0 + lane;
-          pid = bj < nblk ? block_page(si, hrow, lrow, itm.blk_begin + bj) : 0;
+          pid = bj < nblk ? block_page(si, hrow, lrow, blk0 + bj) : 0;
         }
         const int st = n % TC_STAGES;
         int ok = 1;
-        if (lane == 0) ok = mbar_wait(d, &bars[B_KV_EMPTY + st], ((n / TC_STAGES) & 1) ^ 1);
+        if (lane == 0) ok = mbar_wait(d, &bars[b_empty + st], ((n / TC_STAGES) & 1) ^ 1);
         ok = __shfl_sync(FULL, ok, 0);
         if (!ok) {
           if (lane == 0) s_abort = 1;
@@ -270,44 +297,43 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
 #pragma unroll
         for (int pg = 0; pg < 4; ++pg) pages[pg] = __shfl_sync(FULL, pid, (b0 & 31) + pg);
         if (lane == 0) {
-          mbar_arrive_expect_tx(&bars[B_KV_FULL + st], npg * 4 * 2048);
-          uint8_t* base = smem + OFF_KV + st * STAGE;
+          mbar_arrive_expect_tx(&bars[b_full + st], npg * 2 * 2048);
+          uint8_t* base = smem + OFF_KV + st * STAGE + (is_v ? 2 * KV_PANEL : 0);
           for (int pg = 0; pg < npg; ++pg) {
-            const int rk = (((pages[pg] * L + layer) * 2 + 0) * H + head) * PS;
-            const int rv = rk + H * PS;
-            tma_load_2d(base + 0 * KV_PANEL + pg * 2048, &map_lo, 0, rk, &bars[B_KV_FULL + st]);
-            tma_load_2d(base + 1 * KV_PANEL + pg * 2048, &map_hi, 0, rk, &bars[B_KV_FULL + st]);
-            tma_load_2d(base + 2 * KV_PANEL + pg * 2048, &map_lo, 0, rv, &bars[B_KV_FULL + st]);
-            tma_load_2d(base + 3 * KV_PANEL + pg * 2048, &map_hi, 0, rv, &bars[B_KV_FULL + st]);
+            // Pool rows of this page's K (kv = 0) or V (kv = 1) tile of `head`.
+            const int row = (((pages[pg] * L + layer) * 2 + (is_v ? 1 : 0)) * H + head) * PS;
+            tma_load_2d(base + pg * 2048, &map_lo, 0, row, &bars[b_full + st]);
+            tma_load_2d(base + KV_PANEL + pg * 2048, &map_hi, 0, row, &bars[b_full + st]);
           }
         }
       }
       stop = stop || __any_sync(FULL, s_abort != 0);
     }
-  } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
+  } else if (warp == 1 || warp == 7) {
+    // ---------------- MMA issuers ----------------
+    // One elected thread each: warp 1 issues S = Q K^T of every stage, warp 7
+    // O += P V.  Their products use different accumulators, and each thread's
+    // tcgen05.commit tracks only its own MMAs, so the two streams interleave in
+    // the tensor pipe and neither waits behind the other's issue cost.
     if (lane == 0) {
-      constexpr uint32_t ID_S = instr_desc(NK, M, false);
-      constexpr uint32_t ID_PV = instr_desc(D, M, true);
-      uint32_t n = 0;      // K/V stages consumed
-      uint32_t sc = 0;     // S tiles issued
-      uint32_t pv = 0;     // P V products issued
-      uint32_t items = 0;  // items started
-      for (int it = blockIdx.x; it < n_items && !s_abort; it += gridDim.x, ++items) {
-        const Item itm = d.pf_items[it / H];
-        const int nblk = itm.blk_end - itm.blk_begin;
-        const int n_st = (nblk + 3) / 4;
-        if (!mbar_wait(d, &bars[B_Q], items & 1)) {
-          s_abort = 1;
-          break;
-        }
-        tc_fence_after();
-        // S(k) is issued before P(k-1) V(k-1) so the softmax of stage k overlaps it.
-        for (int k = 0; k <= n_st && !s_abort; ++k) {
-          if (k < n_st) {
+      uint32_t n = 0;  // K/V stages of the earlier segments
+      if (warp == 1) {
+        constexpr uint32_t ID_S = instr_desc(NK, M, false);
+        uint32_t sc = 0;     // S tiles issued
+        uint32_t segs = 0;   // segments started
+        for (int u = u_begin; u < u_end && !s_abort; ++segs) {
+          const UnitSeg seg = unit_segment(d, u, u_end);
+          u = seg.end;
+          const int n_st = (seg.end - seg.u + 3) / 4;
+          if (!mbar_wait(d, &bars[B_Q], segs & 1)) {
+            s_abort = 1;
+            break;
+          }
+          tc_fence_after();
+          for (int k = 0; k < n_st && !s_abort; ++k) {
             const int st = (n + k) % TC_STAGES;
             const int sb = sc % 2;
-            if (!mbar_wait(d, &bars[B_KV_FULL + st], ((n + k) / TC_STAGES) & 1) ||
+            if (!mbar_wait(d, &bars[B_K_FULL + st], ((n + k) / TC_STAGES) & 1) ||
                 !mbar_wait(d, &bars[B_S_EMPTY + sb], ((sc / 2) & 1) ^ 1)) {
               s_abort = 1;
               break;
@@ -316,39 +342,50 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
             const uint32_t kbase = sKV + st * STAGE;
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t qa = sQ + (kk >> 2) * Q_PANEL + (kk & 3) * 32;
+              // 16 dims per step: 8 TMEM columns of Q; 32 bytes of a swizzled K row.
               const uint32_t kb = kbase + (kk >> 2) * KV_PANEL + (kk & 3) * 32;
-              tc_mma(tmem + S_COL + sb * NK, smem_desc(qa, 0, 1024), smem_desc(kb, 0, 1024),
-                     ID_S, kk > 0 ? 1u : 0u);
+              tc_mma_ts(tmem + S_COL + sb * NK, tmem + Q_COL + kk * 8, smem_desc(kb, 0, 1024),
+                        ID_S, kk > 0 ? 1u : 0u);
             }
             tc_commit(&bars[B_S_FULL + sb]);
+            tc_commit(&bars[B_K_EMPTY + st]);
             ++sc;
           }
-          if (k >= 1) {
-            const int kp = k - 1;
-            const int st = (n + kp) % TC_STAGES;
+          n += n_st;
+        }
+      } else {
+        constexpr uint32_t ID_PV = instr_desc(D, M, true);
+        uint32_t pv = 0;  // P V products issued
+        for (int u = u_begin; u < u_end && !s_abort;) {
+          const UnitSeg seg = unit_segment(d, u, u_end);
+          u = seg.end;
+          const int n_st = (seg.end - seg.u + 3) / 4;
+          for (int k = 0; k < n_st && !s_abort; ++k) {
+            const int st = (n + k) % TC_STAGES;
             const int pb = pv % 2;
-            if (!mbar_wait(d, &bars[B_P_FULL + pb], (pv / 2) & 1)) {
+            if (!mbar_wait(d, &bars[B_V_FULL + st], ((n + k) / TC_STAGES) & 1) ||
+                !mbar_wait(d, &bars[B_P_FULL + pb], (pv / 2) & 1)) {
               s_abort = 1;
               break;
             }
             tc_fence_after();
             const uint32_t vbase = sKV + st * STAGE + 2 * KV_PANEL;
-            const uint32_t pbase = sP + pb * P_BYTES;
 #pragma unroll
             for (int kk = 0; kk < NK / 16; ++kk) {
-              const uint32_t pa = pbase + kk * 32;
+              // 16 keys per step: 8 TMEM columns of P; 16 rows of the V panels.  The
+              // first product of a segment overwrites O (its previous contents were
+              // read by the epilogue before this segment's first P was written).
               const uint32_t vb = vbase + kk * 16 * 128;
-              tc_mma(tmem + O_COL, smem_desc(pa, 0, 1024), smem_desc(vb, KV_PANEL, 1024), ID_PV,
-                     (kp > 0 || kk > 0) ? 1u : 0u);
+              tc_mma_ts(tmem + O_COL, tmem + P_COL + pb * (NK / 2) + kk * 8,
+                        smem_desc(vb, KV_PANEL, 1024), ID_PV, (k > 0 || kk > 0) ? 1u : 0u);
             }
-            tc_commit(&bars[B_KV_EMPTY + st]);
+            tc_commit(&bars[B_V_EMPTY + st]);
             tc_commit(&bars[B_P_EMPTY + pb]);
-            tc_commit(&bars[B_O]);
+            tc_commit(&bars[B_O + pb]);
             ++pv;
           }
+          n += n_st;
         }
-        n += n_st;
       }
       // No MMA may still be running when the tensor memory is released.
       tc_commit(&bars[B_FINAL]);
@@ -370,47 +407,53 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       dead = !__all_sync(FULL, mbar_wait(d, bar, parity));
       if (dead && lane == 0) s_abort = 1;
     };
-    for (int it = blockIdx.x; it < n_items; it += gridDim.x) {
-      const int item = it / H, head = it % H;
-      const Item itm = d.pf_items[item];
-      const SeqInfo si = d.seq[itm.seq];
-      const int32_t* hrow = d.hist_pt + (size_t)si.sid * d.max_pages_per_session;
-      const int32_t* lrow = d.live_pt + (size_t)si.sid * d.max_pages_per_session;
-      const int nblk = itm.blk_end - itm.blk_begin;
+    for (int u = u_begin; u < u_end;) {
+      const UnitSeg seg = unit_segment(d, u, u_end);
+      const int first = seg.u == u_begin;
+      u = seg.end;
+      const int head = seg.head;
+      const SeqInfo& si = seg.si;
+      const int blk0 = seg.blk_begin(), nblk = seg.end - seg.u;
       const int n_st = (nblk + 3) / 4;
       const int R = si.t * G;
       const bool live = r < R;
       const int t = r / G, g = r % G;
       const int qlog = si.n_hist + si.n_live - si.t + t;
-      // The previous item's products are complete (its epilogue waited for the
-      // last one), so the query tile can be overwritten.
-      if (live && !dead) {
-        // Chunk c (dims 8c..8c+7) of the first half pairs with chunk c of the second.
-        const uint4* qrow = reinterpret_cast<const uint4*>(
-            q + ((size_t)(si.q_row0 + t) * d.q_heads + head * G + g) * D);
-        const float4* cs = reinterpret_cast<const float4*>(d.rope + (size_t)(si.pos_first + t) * (D / 2));
-#pragma unroll 2
-        for (int c = 0; c < 8; ++c) {
-          const uint4 wa = qrow[c], wb = qrow[c + 8];
-          const uint32_t ua[4] = {wa.x, wa.y, wa.z, wa.w}, ub[4] = {wb.x, wb.y, wb.z, wb.w};
-          float ya[8], yb[8];
+      // The previous segment's products are complete (its epilogue waited for the
+      // last one), so the query tile in tensor memory can be overwritten.  Every
+      // lane writes its row: the query (bfloat16 pairs, dims 0..127 in columns
+      // 0..63), or zeros for padding rows.
+      if (!dead) {
+        uint32_t qw[D / 2];
+        if (live) {
+          // Chunk c (dims 8c..8c+7) of the first half pairs with chunk c of the second.
+          const uint4* qrow = reinterpret_cast<const uint4*>(
+              q + ((size_t)(si.q_row0 + t) * d.q_heads + head * G + g) * D);
+          const float4* cs =
+              reinterpret_cast<const float4*>(d.rope + (size_t)(si.pos_first + t) * (D / 2));
 #pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const float4 t4 = cs[c * 4 + h];  // (cos, sin) of dims 8c + 2h, 8c + 2h + 1
-            const float a0 = bf16lo(ua[h]), a1 = bf16hi(ua[h]);
-            const float b0 = bf16lo(ub[h]), b1 = bf16hi(ub[h]);
-            ya[2 * h] = fmaf(a0, t4.x, -b0 * t4.y) * qk_scale;
-            yb[2 * h] = fmaf(b0, t4.x, a0 * t4.y) * qk_scale;
-            ya[2 * h + 1] = fmaf(a1, t4.z, -b1 * t4.w) * qk_scale;
-            yb[2 * h + 1] = fmaf(b1, t4.z, a1 * t4.w) * qk_scale;
+          for (int c = 0; c < 8; ++c) {
+            const uint4 wa = qrow[c], wb = qrow[c + 8];
+            const uint32_t ua[4] = {wa.x, wa.y, wa.z, wa.w}, ub[4] = {wb.x, wb.y, wb.z, wb.w};
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const float4 t4 = cs[c * 4 + h];  // (cos, sin) of dims 8c + 2h, 8c + 2h + 1
+              const float a0 = bf16lo(ua[h]), a1 = bf16hi(ua[h]);
+              const float b0 = bf16lo(ub[h]), b1 = bf16hi(ub[h]);
+              qw[4 * c + h] = pack_bf16(fmaf(a0, t4.x, -b0 * t4.y) * qk_scale,
+                                        fmaf(a1, t4.z, -b1 * t4.w) * qk_scale);
+              qw[D / 4 + 4 * c + h] = pack_bf16(fmaf(b0, t4.x, a0 * t4.y) * qk_scale,
+                                                fmaf(b1, t4.z, a1 * t4.w) * qk_scale);
+            }
           }
-          st_shared_v4(sw128(sQ, r, c), pack_bf16(ya[0], ya[1]), pack_bf16(ya[2], ya[3]),
-                       pack_bf16(ya[4], ya[5]), pack_bf16(ya[6], ya[7]));
-          st_shared_v4(sw128(sQ + Q_PANEL, r, c), pack_bf16(yb[0], yb[1]), pack_bf16(yb[2], yb[3]),
-                       pack_bf16(yb[4], yb[5]), pack_bf16(yb[6], yb[7]));
+        } else {
+#pragma unroll
+          for (int j = 0; j < D / 2; ++j) qw[j] = 0u;
         }
+        tmem_st32(trow + Q_COL, qw);
+        tmem_st32(trow + Q_COL + 32, qw + 32);
       }
-      fence_proxy_async_smem();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars[B_Q]);
 
@@ -435,7 +478,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
         bool interior = npg == 4;
 #pragma unroll
         for (int pg = 0; pg < 4; ++pg) {
-          brs[pg] = block_range(si, itm.blk_begin + 4 * k + min(pg, npg - 1));
+          brs[pg] = block_range(si, blk0 + 4 * k + min(pg, npg - 1));
           interior = interior && brs[pg].lo == 0 && brs[pg].hi == PS;
         }
         interior = interior && brs[3].base + PS - 1 <= si.n_hist + si.n_live - si.t;
@@ -461,7 +504,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
         const bool need = mx > m_used + RESCALE_LOG2;
         const bool have_o = pv > 0 && m_used != -INFINITY;
         if (__any_sync(FULL, need && have_o)) {
-          wait(&bars[B_O], (pv - 1) & 1);
+          wait(&bars[B_O + (pv - 1) % 2], ((pv - 1) / 2) & 1);
           tc_fence_after();
           const float f = (need && have_o) ? exp2f(m_used - mx) : 1.f;
 #pragma unroll
@@ -478,7 +521,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
           if (have_o) l *= exp2f(m_used - mx);
           m_used = mx;
         }
-        // P = exp2(s - m_used) as bfloat16 into P buffer pb (row r, 64 keys = 128 B).
+        // P = exp2(s - m_used) as bfloat16 pairs into TMEM buffer pb (row r, 32 columns).
         wait(&bars[B_P_EMPTY + pb], ((pv / 2) & 1) ^ 1);
         // Masked keys are -inf and give 0; a row with no finite key yet uses 0 as
         // its reference so that no -inf - -inf appears; padding rows get weight 0.
@@ -493,20 +536,17 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
           pw[j / 2] = pack_bf16(p0, p1);
         }
         l += rs0 + rs1;
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          st_shared_v4(sw128(sP + pb * P_BYTES, r, c), pw[4 * c], pw[4 * c + 1], pw[4 * c + 2],
-                       pw[4 * c + 3]);
-        fence_proxy_async_smem();
+        if (!dead) tmem_st32(trow + P_COL + pb * (NK / 2), pw);
+        tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars[B_P_FULL + pb]);
         ++pv;
       }
       // Epilogue: wait for the last P V, read O.
-      wait(&bars[B_O], (pv - 1) & 1);
+      wait(&bars[B_O + (pv - 1) % 2], ((pv - 1) / 2) & 1);
       tc_fence_after();
-      const bool single = si.pf_chunks == 1;
-      const int slot = (si.pf_base + itm.chunk) * H + head;
+      const bool single = seg.whole();
+      const int slot = 2 * cta + (first ? 0 : 1);
       const size_t prow0 = (size_t)slot * (PF_MAX_TOKENS * G) + r;
       const bool write = live && !dead;
       const float inv = 1.f / l;
@@ -533,28 +573,26 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       }
       tc_fence_before();
       if (!single) {
-        // Split-K: publish this chunk's (O, max, sum); the last CTA to arrive for the
-        // (session, head) merges every chunk, one thread per query row.  All four
-        // softmax warps reach both named barriers on every such item.
+        // Split-K: publish this part's (O, max, sum); the last CTA to arrive for the
+        // (session, head) merges every part, one thread per query row.  All four
+        // softmax warps reach both named barriers on every such segment.
         if (write) d.pf_part_ml[prow0] = make_float2(m_used, l);
-        __threadfence();
+        const int cf = us.owner(seg.pair_start), nch = us.owner(seg.pair_end - 1) - cf + 1;
         asm volatile("bar.sync 1, 128;" ::: "memory");
-        if (warp == 2 && lane == 0) {
-          const int old = atomicAdd(&d.pf_count[itm.seq * H + head], 1);
-          s_last = (old == si.pf_chunks - 1);
-        }
+        if (warp == 2 && lane == 0)
+          s_last = arrive_acq_rel(&d.pf_count[seg.seq * H + head], nch);
         asm volatile("bar.sync 1, 128;" ::: "memory");
         if (s_last) {
-          __threadfence();
           if (live) {
-            const size_t s0 = (size_t)(si.pf_base * H + head) * (PF_MAX_TOKENS * G) + r;
-            const size_t cstride = (size_t)H * (PF_MAX_TOKENS * G);
+            const int first_slot = us.slot_of(cf, cf, seg.pair_start);
+            auto prow = [&](int ch) {
+              return (size_t)(ch ? 2 * (cf + ch) : first_slot) * (PF_MAX_TOKENS * G) + r;
+            };
             float Mx = -INFINITY;
-            for (int ch = 0; ch < si.pf_chunks; ++ch)
-              Mx = fmaxf(Mx, __ldcg(&d.pf_part_ml[s0 + ch * cstride]).x);
+            for (int ch = 0; ch < nch; ++ch) Mx = fmaxf(Mx, __ldcg(&d.pf_part_ml[prow(ch)]).x);
             float Ls = 0.f;
-            for (int ch = 0; ch < si.pf_chunks; ++ch) {
-              const float2 ml = __ldcg(&d.pf_part_ml[s0 + ch * cstride]);
+            for (int ch = 0; ch < nch; ++ch) {
+              const float2 ml = __ldcg(&d.pf_part_ml[prow(ch)]);
               Ls += ml.y * exp2_safe(ml.x, Mx);
             }
             const float invL = 1.f / Ls;
@@ -564,8 +602,8 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
               float acc[32];
 #pragma unroll
               for (int i = 0; i < 32; ++i) acc[i] = 0.f;
-              for (int ch = 0; ch < si.pf_chunks; ++ch) {
-                const size_t row = s0 + ch * cstride;
+              for (int ch = 0; ch < nch; ++ch) {
+                const size_t row = prow(ch);
                 const float sc2 = exp2_safe(__ldcg(&d.pf_part_ml[row]).x, Mx) * invL;
                 const float4* src =
                     reinterpret_cast<const float4*>(d.pf_part_o + row * D + c * 32);
@@ -586,7 +624,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
                                pack_bf16(acc[i + 6], acc[i + 7]));
             }
           }
-          if (warp == 2 && lane == 0) d.pf_count[itm.seq * H + head] = 0;
+          if (warp == 2 && lane == 0) d.pf_count[seg.seq * H + head] = 0;
         }
       }
     }

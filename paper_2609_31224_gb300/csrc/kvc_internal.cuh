@@ -45,8 +45,8 @@ struct SeqInfo {
   int32_t live_head;
   int32_t n_live;
   int32_t n_blocks;     // n_hist_pages + n_live_pages
-  int32_t dec_chunks;   // unused by decode (stream-K split)
-  int32_t dec_base;     // first decode unit (session, kv head, page) of this session
+  int32_t dec_chunks;   // unused (attention splits the call's units, see UnitSplit)
+  int32_t unit_base;    // first (session, kv head, page) unit of this session
   int32_t pf_chunks;
   int32_t pf_base;
   int32_t pad[3];
@@ -65,11 +65,11 @@ struct DevGlobals {
   int32_t err;
   int32_t n_seq;
   int64_t pages_used;
-  int32_t n_dec_items;
+  int32_t n_units;
   int32_t n_pf_items;
   int32_t n_moves;
   int32_t total_tokens;
-  int32_t dec_nb_max;   // largest n_blocks among the last append's sessions
+  int32_t nb_max;   // largest n_blocks among the last append's sessions
   int32_t pad[7];
 };
 
@@ -144,6 +144,78 @@ __device__ inline BlockRef block_ref(const SeqInfo& si, const int32_t* hist_row,
     r.base = si.n_hist + s0 - si.live_head;
   }
   return r;
+}
+
+// ---------------------------------------------------------------------------
+// Stream-K split of an attention call's (session, KV head, page) units.  Units
+// are ordered session-major, then head, then page; seq[i].unit_base is session
+// i's first.  The U units are cut into n_cta equal contiguous ranges, one per
+// CTA.  A range covers "segments", the parts of (session, head) pairs inside it;
+// only its first and last segments can be partial, and their partial states go
+// to slots 2c and 2c + 1.  The CTAs owner(pair_start) .. owner(pair_end - 1)
+// share a pair, and the last of them to finish merges it.
+// ---------------------------------------------------------------------------
+struct UnitSplit {
+  int U, n_cta;
+  __device__ int start_of(int c) const { return (int)((int64_t)c * U / n_cta); }
+  __device__ int owner(int64_t u) const { return (int)(((u + 1) * n_cta - 1) / U); }
+  // Slot of CTA cc's part of a pair whose first CTA is cf: cc's first segment,
+  // except in cf when the pair begins after the start of cf's range.
+  __device__ int slot_of(int cc, int cf, int pair_start) const {
+    return cc != cf ? 2 * cc : (start_of(cf) != pair_start ? 2 * cf + 1 : 2 * cf);
+  }
+};
+
+// At most `grid` CTAs, at least `min_units` units each, and few enough that no
+// pair spans more than `max_parts` CTAs.
+__device__ inline UnitSplit unit_split(const Dev& d, int grid, int min_units, int max_parts) {
+  UnitSplit s;
+  s.U = d.g->n_units;
+  const int nb_max = max(1, d.g->nb_max);
+  const int c_parts = (int)((int64_t)s.U * (max_parts - 2) / (nb_max + max_parts - 2));
+  s.n_cta = max(1, min(grid, min((s.U + min_units - 1) / min_units, c_parts)));
+  return s;
+}
+
+struct UnitSeg {
+  int seq, head;             // session of the call, KV head
+  int pair_start, pair_end;  // the pair's units
+  int u, end;                // this segment's units [u, end)
+  SeqInfo si;
+  __device__ int blk_begin() const { return u - pair_start; }
+  __device__ int blk_end() const { return end - pair_start; }
+  __device__ bool whole() const { return u == pair_start && end == pair_end; }
+};
+
+// The segment that starts at unit u of a range ending at u_end.
+__device__ inline UnitSeg unit_segment(const Dev& d, int u, int u_end) {
+  int lo = 0, hi = d.g->n_seq - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (d.seq[mid].unit_base <= u) lo = mid;
+    else hi = mid - 1;
+  }
+  UnitSeg s;
+  s.seq = lo;
+  s.si = d.seq[lo];
+  const int nb = s.si.n_blocks;
+  s.head = (u - s.si.unit_base) / nb;
+  s.pair_start = s.si.unit_base + s.head * nb;
+  s.pair_end = s.pair_start + nb;
+  s.u = u;
+  s.end = min(u_end, s.pair_end);
+  return s;
+}
+
+// Arrive at a pair's counter once this CTA's partial state is written; true in
+// the last of `parts` arrivals.  The caller synchronises the participating
+// threads before (so that their partial writes precede the arrival) and after
+// (so that, in the last CTA, the loads of the other parts follow it); one
+// thread's acquire-release atomic then publishes and acquires at GPU scope.
+__device__ inline bool arrive_acq_rel(int* counter, int parts) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(counter) : "memory");
+  return old == parts - 1;
 }
 
 // Valid slot range [lo, hi) and logical base of virtual block b, without

@@ -165,8 +165,7 @@ __global__ void init_rope_kernel(Dev d, double base) {
 // split-K work lists of the attention calls that follow.
 // ---------------------------------------------------------------------------
 __device__ void build_worklist(const Dev& d, int n_seq, int nb, int target, int min_blocks,
-                               int max_items, Item* items, bool decode, int* s_warp,
-                               int* s_total_items) {
+                               int max_items, Item* items, int* s_warp, int* s_total_items) {
   const int i = threadIdx.x;
   int total_blocks;
   (void)block_exclusive_scan(i < n_seq ? nb : 0, &total_blocks, s_warp);
@@ -180,13 +179,8 @@ __device__ void build_worklist(const Dev& d, int n_seq, int nb, int target, int 
   }
   if (i < n_seq) {
     SeqInfo& si = d.seq[i];
-    if (decode) {
-      si.dec_chunks = chunks;
-      si.dec_base = base;
-    } else {
-      si.pf_chunks = chunks;
-      si.pf_base = base;
-    }
+    si.pf_chunks = chunks;
+    si.pf_base = base;
     for (int c = 0; c < chunks; ++c) {
       Item it;
       it.seq = i;
@@ -204,7 +198,7 @@ __device__ void build_worklist(const Dev& d, int n_seq, int nb, int target, int 
 // attention kernels nothing to do.
 __device__ void abandon_append(const Dev& d) {
   d.g->total_tokens = 0;
-  d.g->n_dec_items = 0;
+  d.g->n_units = 0;
   d.g->n_pf_items = 0;
 }
 
@@ -312,26 +306,27 @@ __global__ void __launch_bounds__(META_THREADS) append_plan_kernel(Dev d, Append
     d.seq[i] = si;
   }
   __syncthreads();
-  // 4. Split-K work lists for decode and prefill attention.
-  // Decode splits the call's (session, kv head, page) units evenly over its CTAs
-  // (stream-K); it needs each session's first unit, the total and the largest session.
+  // 4. Split-K work for the attention calls.  The decode and bfloat16 prefill
+  // kernels split the call's (session, kv head, page) units evenly over their CTAs
+  // (stream-K): they need each session's first unit, the total and the largest
+  // session.  The binary32 prefill kernel takes the per-session chunk list.
   {
     int total_units;
     const int ubase = block_exclusive_scan(i < n_seq ? nb * d.kv_heads : 0, &total_units, s_warp);
     const int nb_max = block_max(i < n_seq ? nb : 0, s_warp);
-    if (i < n_seq) d.seq[i].dec_base = ubase;
+    if (i < n_seq) d.seq[i].unit_base = ubase;
     if (i == 0) {
       s_total_dec = total_units;
-      d.g->dec_nb_max = nb_max;
+      d.g->nb_max = nb_max;
     }
     __syncthreads();
   }
-  build_worklist(d, n_seq, nb, a.pf_target, a.pf_min_blocks, d.max_pf_items, d.pf_items, false,
-                 s_warp, &s_total_pf);
+  build_worklist(d, n_seq, nb, a.pf_target, a.pf_min_blocks, d.max_pf_items, d.pf_items, s_warp,
+                 &s_total_pf);
   if (i == 0) {
     d.g->n_seq = n_seq;
     d.g->total_tokens = a.total;
-    d.g->n_dec_items = s_total_dec;
+    d.g->n_units = s_total_dec;
     d.g->n_pf_items = s_total_pf;
     d.g->pages_used += total_need;
   }
