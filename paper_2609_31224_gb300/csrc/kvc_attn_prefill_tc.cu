@@ -457,6 +457,15 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars[B_Q]);
 
+      // Blocks that may need a mask: the partly filled last history page, the
+      // first live page when it starts mid-page, and every block from the one
+      // holding the chunk's first query on (causal).  A stage of four pages that
+      // avoids them all is interior.
+      const int nhp = si.n_hist_pages;
+      const int b_hist_part = (si.n_hist % PS) ? nhp - 1 : -PS;
+      const int b_live_part = si.live_head ? nhp : -PS;
+      const int sl_first = si.live_head + si.n_live - si.t;  // live slot of the first query
+      const int b_causal = nhp + sl_first / PS + ((sl_first % PS) == PS - 1 ? 1 : 0);
       float m_used = -INFINITY, l = 0.f;
       for (int k = 0; k < n_st; ++k) {
         const int sb = sc % 2, pb = pv % 2;
@@ -474,15 +483,13 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
         // query) need no mask.  Padding rows (r >= T*G) are left unmasked: their
         // products stay finite and their outputs are never written.
         const int npg = min(4, nblk - 4 * k);
-        BlockRange brs[4];
-        bool interior = npg == 4;
-#pragma unroll
-        for (int pg = 0; pg < 4; ++pg) {
-          brs[pg] = block_range(si, blk0 + 4 * k + min(pg, npg - 1));
-          interior = interior && brs[pg].lo == 0 && brs[pg].hi == PS;
-        }
-        interior = interior && brs[3].base + PS - 1 <= si.n_hist + si.n_live - si.t;
+        const int b0 = blk0 + 4 * k;
+        const bool interior = npg == 4 && b0 + 3 < b_causal &&
+                              (unsigned)(b_hist_part - b0) > 3u && (unsigned)(b_live_part - b0) > 3u;
         if (!interior) {
+          BlockRange brs[4];
+#pragma unroll
+          for (int pg = 0; pg < 4; ++pg) brs[pg] = block_range(si, b0 + min(pg, npg - 1));
 #pragma unroll
           for (int pg = 0; pg < 4; ++pg) {
 #pragma unroll
@@ -494,9 +501,14 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
             }
           }
         }
-        float mx = -INFINITY;
+        // Row maximum over 8 independent chains.
+        float m8[8];
 #pragma unroll
-        for (int j = 0; j < NK; ++j) mx = fmaxf(mx, s[j]);
+        for (int i = 0; i < 8; ++i) m8[i] = s[i];
+#pragma unroll
+        for (int j = 8; j < NK; ++j) m8[j % 8] = fmaxf(m8[j % 8], s[j]);
+        float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                         fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
         if (dead || !live) mx = -INFINITY;
         // Rescale O (in TMEM) and l only when the row maximum grows by > 2^8; this
         // waits for the previous P V product.  Every lane of the warp takes part
@@ -526,16 +538,16 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
         // Masked keys are -inf and give 0; a row with no finite key yet uses 0 as
         // its reference so that no -inf - -inf appears; padding rows get weight 0.
         const float mref = !live ? INFINITY : (m_used == -INFINITY ? 0.f : m_used);
-        float rs0 = 0.f, rs1 = 0.f;
+        float rs[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         uint32_t pw[NK / 2];
 #pragma unroll
         for (int j = 0; j < NK; j += 2) {
           const float p0 = ex2(s[j] - mref), p1 = ex2(s[j + 1] - mref);
-          rs0 += p0;
-          rs1 += p1;
+          rs[j % 8] += p0;
+          rs[j % 8 + 1] += p1;
           pw[j / 2] = pack_bf16(p0, p1);
         }
-        l += rs0 + rs1;
+        l += ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
         if (!dead) tmem_st32(trow + P_COL + pb * (NK / 2), pw);
         tc_fence_before();
         __syncwarp();
