@@ -18,6 +18,7 @@ collective on the data path): weak scaling.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -33,6 +34,29 @@ sys.path.insert(0, ROOT)
 
 METRIC = "audio-seconds processed/sec (evict+attn, all layers); HBM GB/s vs GB300 peak"
 UNIT = "audio-s/s"
+
+
+# DRAM bytes per algorithmic byte of the roofline kernel (reads + writes), from one
+# ncu capture of the 16-session, two-layer reduced case: 275.30 MB of traffic for a
+# 269.29 MB launch.  Valid only while the decode sources hash to the version it was
+# taken on; the roofline's traffic is null otherwise.
+DECODE_TRAFFIC_RATIO = 275.30 / 269.29
+DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
+                          "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
+DECODE_TRAFFIC_SHA256 = "ef88ea5f45197e0a7a0615a9ab72eea358e6cdb1da904905c924c575b0428cd0"
+
+
+def decode_traffic(alg_bytes_per_launch):
+    """Per-launch DRAM traffic of the decode kernel, scaled from the capture, or None."""
+    if not alg_bytes_per_launch:
+        return None
+    h = hashlib.sha256()
+    for f in DECODE_TRAFFIC_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    if h.hexdigest() != DECODE_TRAFFIC_SHA256:
+        return None
+    return DECODE_TRAFFIC_RATIO * alg_bytes_per_launch
 
 
 def load_peaks():
@@ -263,7 +287,9 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "peak_kind": f"{peak_kind} copy bandwidth",
             "unit": "GB/s",
             "frac": (dec_gbs / peak) if dec_gbs else None,
-            "traffic": None,
+            "traffic": decode_traffic((sum(dec_bytes) / len(dec_bytes)) if dec_bytes else None),
+            "traffic_note": "ncu DRAM bytes per algorithmic byte on the 16-session reduced "
+                            "case, scaled to this launch",
             "algorithmic_bytes_per_launch": (sum(dec_bytes) / len(dec_bytes)) if dec_bytes else None,
             "avg_launch_us": (1e3 * sum(dec_times) / len(dec_times)) if dec_times else None,
         },
