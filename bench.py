@@ -164,7 +164,9 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     start = args.start if args.start is not None else S.steady_state_step(w, scripts)
     n_steps_total = len(drv.sched)
     assert start - args.warmup >= 0 and start + args.steps <= n_steps_total
-    e2e_steps = args.e2e_steps if args.e2e_steps is not None else min(args.steps, 8)
+    # As many end-to-end steps as timed steps: step cost varies with the decode rounds
+    # (speaking turns), so a shorter window would not be comparable.
+    e2e_steps = args.e2e_steps if args.e2e_steps is not None else args.steps
     assert start + args.steps + e2e_steps <= n_steps_total
 
     # 1. Bring the cache to the step before the warm-up (append + evict only).
@@ -304,6 +306,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
 def run_e2e(drv, w, n_steps: int, world: int) -> dict:
     import torch
     stream = torch.cuda.current_stream()
+    first_step = drv.step_index
     steps = [drv.prepare_step() for _ in range(n_steps)]
     # Move every input to pinned host memory; keep same-shaped device buffers.
     host, dev = [], []
@@ -363,7 +366,7 @@ def run_e2e(drv, w, n_steps: int, world: int) -> dict:
     audio_s = sum(len(st.pairs) for st in steps)
     return {"value": world * audio_s / (ms / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d_total / n_steps, "d2h_bytes_per_step": d2h_total / n_steps,
-            "steps": n_steps, "host_wall_s": wall}
+            "steps": n_steps, "first_step": first_step, "host_wall_s": wall}
 
 
 # -- the oracle on the host cores -----------------------------------------------------------------
