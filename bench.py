@@ -369,6 +369,50 @@ def run_e2e(drv, w, n_steps: int, world: int) -> dict:
             "steps": n_steps, "first_step": first_step, "host_wall_s": wall}
 
 
+# -- budget versus no budget on one session ---------------------------------------------------
+def run_unbounded_comparison() -> dict:
+    """The single-session workload with B = 4096 and with B = infinity, on the same seeded
+    inputs, through all 600 units: peak resident positions and K/V bytes, and the summed
+    GPU time of every attention call (events from the end of each call's append to its
+    last layer)."""
+    import torch
+    from synth import script as S
+    from synth.driver import Driver
+    res = {}
+    for w in (S.SINGLE_BF16, S.SINGLE_BF16_UNBOUNDED):
+        scripts = S.workload_scripts(w)
+        drv = Driver(w, scripts)
+        spans = []
+        for _ in range(len(drv.sched)):
+            st = drv.prepare_step()
+            for c in st.calls:
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                drv.run_call(c, on_append=lambda _c, e=e0: e.record())
+                e1.record()
+                if c.kind != "prefix":
+                    spans.append((e0, e1))
+            drv.cache.evict(st.evict_sessions, drv.resident_out)
+            del st
+        torch.cuda.synchronize()
+        info = drv.cache.export_state(0)
+        res[w.name] = {
+            "budget": w.budget,
+            "attention_ms": sum(a.elapsed_time(b) for a, b in spans),
+            "attention_calls": len(spans) * w.layers,
+            "peak_resident_positions": info["peak_resident"],
+            "end_resident_positions": info["resident"],
+            "peak_kv_bytes": info["peak_resident"] * w.kv_bytes_per_position,
+        }
+        del drv
+        torch.cuda.empty_cache()
+    b, f = res[S.SINGLE_BF16.name], res[S.SINGLE_BF16_UNBOUNDED.name]
+    return {"comparison": "single session, B=4096 vs B=infinity, same seeded inputs",
+            "units": S.SINGLE_BF16.units, "runs": res,
+            "peak_kv_reduction": 1.0 - b["peak_kv_bytes"] / f["peak_kv_bytes"],
+            "attention_time_ratio_full_over_budget": f["attention_ms"] / b["attention_ms"]}
+
+
 # -- the oracle on the host cores -----------------------------------------------------------------
 def oracle_sample(layers_sampled: int = 1, session: int = 0, start: int | None = None) -> dict:
     """Time the CPU oracle on one session's unit at the benchmark's steady state, for
@@ -453,6 +497,8 @@ def main():
     ap.add_argument("--start", type=int, default=None, help="first timed step of the schedule")
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--compare-unbounded", action="store_true",
+                    help="print the B=4096 vs B=infinity single-session comparison and exit")
     ap.add_argument("--sessions", type=int, default=None,
                     help="reduced case for profiler captures (default: the full 64)")
     ap.add_argument("--layers", type=int, default=None,
@@ -477,6 +523,10 @@ def main():
 
     from __graft_entry__ import build
     build()
+    if args.compare_unbounded:
+        if rank == 0:
+            print(json.dumps(run_unbounded_comparison()))
+        return
     out = run_ours(args, rank, world, local_rank)
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:

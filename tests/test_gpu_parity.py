@@ -118,6 +118,53 @@ def test_single_session_full_size_metadata_and_sampled_attention():
     assert st["peak_resident"] > 4096
 
 
+def test_single_session_unbounded_full_size():
+    """No-eviction run of the single-session workload (B = infinity): every evict is a
+    no-op checked bit-exact, the cache grows to every fed position (about 13.7K), and
+    attention over the longest contexts is sampled late in the session."""
+    ls, scripts = _lockstep(S.SINGLE_BF16_UNBOUNDED)
+    samples = {0, 300, 598, 599}
+    for step in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda st, kind, i, layer: st in samples and
+                    (layer in (0, 31) or (kind == "decode" and i == 1 and layer == 17)))
+    st = ls.drv.cache.export_state(0)
+    total = len(scripts[0].all_types())
+    assert st["resident"] == total and st["n_evicted"] == 0
+    assert st["peak_resident"] == total > 13000
+    assert ls.n_compared >= 8
+
+
+@pytest.mark.parametrize("budget,window", [(2048, 5), (2048, 20), (8192, 5), (8192, 20)])
+def test_stress_shard(budget, window):
+    """The 256-session stress workload (10-60 minute sessions, 5% units without a segment,
+    2% long segments of 10-30 tokens) at each (B, W) grid point, on a shard of four
+    sessions (one per stride of 64) run until well past the budget: every evict
+    bit-exact, attention sampled at the edges of the run."""
+    w = S.stress256(budget, window)
+    n_units = budget // 20 + 60
+    scripts = []
+    for sid in (3, 67, 131, 195):
+        sc = S.session_script(w, sid)
+        sc.n_transcript = sc.n_transcript[:n_units]
+        sc.n_text = sc.n_text[:n_units]
+        scripts.append(sc)
+    # The shard must exercise both segment edge cases.
+    assert sum(int((sc.n_transcript < 0).sum()) for sc in scripts) > 0
+    assert sum(int((sc.n_transcript >= 10).sum()) for sc in scripts) > 0
+    drv = Driver(w, scripts)
+    ls = Lockstep(drv, w)
+    last = len(drv.sched) - 1
+    samples = {0, last // 2, last - 1, last}
+    for step in range(len(drv.sched)):
+        ls.run_step(attn_pred=lambda st, kind, i, layer: st in samples and layer in (0, 31)
+                    and i in (0, 1, 2))
+    for sc in scripts:
+        st = drv.cache.export_state(sc.session)
+        assert st["n_evicted"] > 0
+        assert st["peak_resident"] > budget
+    assert ls.n_compared >= 16
+
+
 def test_batch64_sampled_at_full_size():
     """64 sessions, offsets U{0..300}: state of every session bit-exact at sampled steps;
     attention of sampled sessions/layers in the launch configuration of the benchmark."""
