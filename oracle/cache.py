@@ -32,12 +32,16 @@ class OracleConfig:
     dtype: str
     rope_base: float
     n_pages: int
+    policy: str = "unit"
+    sink: int = 0
+    recent: int = 0
 
 
 class OracleCache:
     def __init__(self, cfg: OracleConfig):
         self.cfg = cfg
-        self.policy = [SessionPolicy(cfg.budget, cfg.window) for _ in range(cfg.n_sessions)]
+        self.policy = [SessionPolicy(cfg.budget, cfg.window, cfg.policy, cfg.sink, cfg.recent)
+                       for _ in range(cfg.n_sessions)]
         self.layout = [SessionLayout(cfg.page_size) for _ in range(cfg.n_sessions)]
         self.pool = PagePool(cfg.n_pages)
         self.last_append: list[tuple[int, list[int]]] | None = None
@@ -55,10 +59,11 @@ class OracleCache:
         plans = []
         for s in sessions:
             pol, lay = self.policy[s], self.layout[s]
-            units = pol.evict()
-            if units:
-                u_star = units[-1]
-                end = sum(1 for p in lay.live_pos if pol.unit[p] <= u_star)
+            pol.evict()
+            # The live slots whose positions this evict decided form a prefix of the
+            # live region: the survivors among them move to the compacted region.
+            if pol.frontier is not None:
+                end = sum(1 for p in lay.live_pos if p < pol.frontier)
                 survivors = [p for p in lay.live_pos[:end] if not pol.evicted[p]]
             else:
                 end, survivors = 0, []

@@ -263,3 +263,149 @@ def test_layout_invariants_many_sessions(seed):
             slots = {lay.slot_of_logical(i) for i in range(len(st["pos"]))}
             assert len(slots) == len(st["pos"])
         assert used + c.pool.free_count() == total
+
+
+# -- policy variants -------------------------------------------------------------------------
+
+def _brute_force_position_victims(pol, budget, window):
+    """Every set S of resident evictable positions of units 0..unit_cur-W that is
+    oldest-first, brings the count within B (or takes them all) and removes no more
+    than needed; the variant's choice must be the unique such set."""
+    n = pol.pos_next
+    last = pol.unit_cur - window
+    elig = [p for p in range(n) if not pol.evicted[p] and pol.unit[p] >= 0
+            and pol.unit[p] <= last and pol.type[p] in EVICTABLE]
+    r = sum(1 for p in range(n) if not pol.evicted[p])
+    answers = []
+    for k in range(len(elig) + 1):
+        for combo in itertools.combinations(elig, k):
+            s = set(combo)
+            if any(q not in s and q < max(s, default=-1) for q in elig):
+                continue  # not oldest-first
+            fits = budget < 0 or r - len(s) <= budget
+            if budget >= 0 and not (fits or len(s) == len(elig)):
+                continue
+            if budget < 0 and s:
+                continue
+            if s and budget >= 0 and r - (len(s) - 1) <= budget:
+                continue  # one fewer would have been enough
+            answers.append(s)
+    return answers
+
+
+@pytest.mark.parametrize("seed", range(200))
+def test_position_variant_brute_force(seed):
+    rng = np.random.default_rng(1000 + seed)
+    n_units = int(rng.integers(1, 5))
+    budget = int(rng.integers(-1, 12))
+    window = int(rng.integers(0, 4))
+    pol = SessionPolicy(budget, window, policy="position")
+    pol.append([int(rng.choice([ACOUSTIC, TEXT])) for _ in range(int(rng.integers(0, 3)))])
+    for unit in _random_script(rng, n_units, 6):
+        pol.append(unit)
+        answers = _brute_force_position_victims(pol, budget, window)
+        assert len(answers) == 1, answers
+        got = pol.evict()
+        assert set(got) == answers[0] and got == sorted(got)
+        if got:
+            assert pol.frontier == got[-1] + 1
+
+
+@pytest.mark.parametrize("budget,window", [(0, 0), (0, 3), (50, 2), (200, 10), (30, 0)])
+def test_position_variant_invariants(budget, window):
+    for seed in range(6):
+        rng = np.random.default_rng(seed)
+        pol = SessionPolicy(budget, window, policy="position")
+        pol.append([TEXT] * int(rng.integers(0, 5)))
+        for u in range(40):
+            unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * int(rng.integers(0, 20))
+            if rng.random() < 0.8:
+                unit += [ASR_DELIM] + [TRANSCRIPT] * int(rng.poisson(3)) + [ASR_DELIM]
+            pol.append(unit)
+            got = pol.evict()
+            last = pol.unit_cur - window
+            left = [p for p in range(pol.pos_next) if not pol.evicted[p] and pol.unit[p] >= 0
+                    and pol.unit[p] <= last and pol.type[p] in EVICTABLE]
+            # (i) fits in B, or nothing eligible is left
+            if pol.resident() > budget:
+                assert not left
+            # (ii) an evict that removes anything lands exactly on B unless it ran out
+            if got:
+                assert pol.resident() == budget or not left
+            # (iii) only evictable positions of units >= 0 ever go
+            for p in range(pol.pos_next):
+                if pol.evicted[p]:
+                    assert pol.unit[p] >= 0 and pol.type[p] in EVICTABLE
+            # (iv) oldest first: no resident eligible evictable position is older than
+            # an evicted one
+            gone = [p for p in range(pol.pos_next) if pol.evicted[p]]
+            if gone:
+                assert not any(p < gone[-1] for p in left)
+
+
+def test_position_variant_is_finer_than_unit_rule():
+    """Same script, same B and W: the variant keeps at least as many positions after
+    every evict and lands exactly on B whenever it evicts."""
+    rng = np.random.default_rng(5)
+    a = SessionPolicy(300, 3)
+    b = SessionPolicy(300, 3, policy="position")
+    for u in range(60):
+        unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * 16 + [ASR_DELIM] + \
+            [TRANSCRIPT] * int(rng.poisson(3)) + [ASR_DELIM]
+        a.append(unit)
+        b.append(unit)
+        a.evict()
+        got = b.evict()
+        assert b.resident() >= a.resident()
+        if got:
+            assert b.resident() == 300
+
+
+@pytest.mark.parametrize("sink,recent", [(0, 0), (4, 0), (0, 16), (4, 16), (4, 2000), (40, 7)])
+def test_sink_recent_variant_closed_form(sink, recent):
+    rng = np.random.default_rng(sink * 31 + recent)
+    pol = SessionPolicy(-1, 0, policy="sink_recent", sink=sink, recent=recent)
+    pol.append([TEXT] * 3)
+    for u in range(50):
+        unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * int(rng.integers(0, 20)) + \
+            [ASR_DELIM] + [TRANSCRIPT] * int(rng.poisson(3)) + [ASR_DELIM]
+        pol.append(unit)
+        pol.evict()
+        n = pol.pos_next
+        want = [p for p in range(n) if p < sink or p >= n - recent]
+        assert pol.retained_positions() == want
+        assert pol.frontier == max(n - recent, 0)
+
+
+@pytest.mark.parametrize("policy", ["position", "sink_recent"])
+@pytest.mark.parametrize("seed", range(4))
+def test_layout_invariants_policy_variants(policy, seed):
+    rng = np.random.default_rng(seed)
+    n_sessions, ps = 4, 4
+    c = OracleCache(OracleConfig(n_sessions=n_sessions, layers=1, q_heads=1, kv_heads=1,
+                                 head_dim=4, page_size=ps, budget=int(rng.integers(5, 60)),
+                                 window=int(rng.integers(0, 4)), dtype="f32",
+                                 rope_base=10000.0, n_pages=4000, policy=policy, sink=3,
+                                 recent=int(rng.integers(0, 30))))
+    total = c.pool.n_pages
+    for step in range(50):
+        active = sorted(rng.choice(n_sessions, size=int(rng.integers(1, n_sessions + 1)),
+                                   replace=False).tolist())
+        chunks = []
+        for s in active:
+            unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * int(rng.integers(0, 9))
+            unit += [ASR_DELIM] + [TRANSCRIPT] * int(rng.poisson(2)) + [ASR_DELIM]
+            chunks.append(unit)
+        c.append_chunk(active, chunks)
+        c.evict(active)
+        used, seen = 0, set()
+        for s in range(n_sessions):
+            st, lay = c.state(s), c.layout[s]
+            assert st["pos"] == sorted(st["pos"])
+            assert len(lay.hist_pages) == -(-lay.n_hist // ps)
+            assert len(lay.live_pages) == -(-(lay.live_head + lay.n_live) // ps)
+            for pid in lay.hist_pages + lay.live_pages:
+                assert pid not in seen
+                seen.add(pid)
+            used += len(lay.hist_pages) + len(lay.live_pages)
+        assert used + c.pool.free_count() == total
