@@ -54,6 +54,17 @@ enum { KVC_ACOUSTIC = 0, KVC_ASR_DELIM = 1, KVC_TRANSCRIPT = 2, KVC_TEXT = 3 };
  * prefix) and are never evicted. */
 #define KVC_UNIT_BEGIN 0x80
 
+/* Eviction policies.  KVC_POLICY_UNIT is the rule of Sec. 3.3 (the default).
+ * The two others run on the same state for comparison:
+ *  - KVC_POLICY_POSITION: the position-granular reading of the same rule:
+ *    single evictable positions, oldest first, of the units outside the W most
+ *    recent ones, until the resident count fits in B or none is left;
+ *  - KVC_POLICY_SINK_RECENT: the StreamingLLM baseline of Table 1 (footnote:
+ *    attention-sink tokens plus 2,000 recent positions), type-blind: each
+ *    kvc_evict drops every position p with sink <= p < pos_next - recent; B and
+ *    W play no part. */
+enum { KVC_POLICY_UNIT = 0, KVC_POLICY_POSITION = 1, KVC_POLICY_SINK_RECENT = 2 };
+
 /* Status codes. */
 enum {
   KVC_OK = 0,
@@ -89,6 +100,9 @@ typedef struct kvc_config {
   int32_t max_positions;         /* positions fed to one session stay below this */
   int32_t max_seq_per_call;      /* sessions per call, <= 512 */
   int32_t max_tokens_per_call;   /* tokens per kvc_append_chunk call */
+  int32_t policy;                /* KVC_POLICY_*; 0 = the rule of Sec. 3.3 */
+  int32_t sink;                  /* KVC_POLICY_SINK_RECENT: first positions always kept */
+  int32_t recent;                /* KVC_POLICY_SINK_RECENT: most recent positions kept */
 } kvc_config;
 
 /* Supported shapes: (KVC_BF16, head_dim 128) and (KVC_F32, head_dim 64), with
@@ -142,9 +156,11 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions,
 /* Online eviction (Sec. 3.3) for each listed session, run by the caller after
  * a unit: while resident > B, evict the ACOUSTIC and ASR_DELIM positions of
  * the oldest unit u with 0 <= u <= unit_cur - W that still has some; stop
- * when resident <= B or no such unit remains.  Survivors of the consumed
- * live prefix move (all layers, 16-byte copies) to the compacted region in
- * position order; consumed live pages are freed.
+ * when resident <= B or no such unit remains (the variants of KVC_POLICY_*
+ * decide positions instead, see there).  The live slots whose positions the
+ * call decided form a prefix of the live region: its survivors move (all
+ * layers, 16-byte copies) to the compacted region in position order, and
+ * consumed live pages are freed.
  *   d_resident_out  optional device [n_seq] int64: resident count afterwards
  * Invalidates the last append's queries for attention. */
 int kvc_evict(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, int64_t* d_resident_out,

@@ -18,6 +18,9 @@ LIB_PATH = os.path.join(HERE, "libkvc.so")
 KVC_F32, KVC_BF16 = 0, 1
 KVC_ACOUSTIC, KVC_ASR_DELIM, KVC_TRANSCRIPT, KVC_TEXT = 0, 1, 2, 3
 KVC_UNIT_BEGIN = 0x80
+KVC_POLICY_UNIT, KVC_POLICY_POSITION, KVC_POLICY_SINK_RECENT = 0, 1, 2
+POLICIES = {"unit": KVC_POLICY_UNIT, "position": KVC_POLICY_POSITION,
+            "sink_recent": KVC_POLICY_SINK_RECENT}
 STATUS = {0: "KVC_OK", -1: "KVC_EINVAL", -2: "KVC_ENOMEM", -3: "KVC_ECUDA", -4: "KVC_ESTATE",
           -5: "KVC_EDEVICE"}
 
@@ -41,7 +44,8 @@ class Config(ctypes.Structure):
                 ("dtype", ctypes.c_int32), ("rope_base", ctypes.c_double),
                 ("n_pages", ctypes.c_int64), ("max_pages_per_session", ctypes.c_int32),
                 ("max_positions", ctypes.c_int32), ("max_seq_per_call", ctypes.c_int32),
-                ("max_tokens_per_call", ctypes.c_int32)]
+                ("max_tokens_per_call", ctypes.c_int32), ("policy", ctypes.c_int32),
+                ("sink", ctypes.c_int32), ("recent", ctypes.c_int32)]
 
 
 class SessionInfo(ctypes.Structure):
@@ -130,13 +134,14 @@ class KVCache:
                  head_dim: int, budget: int, window: int, dtype: str, n_pages: int,
                  max_pages_per_session: int, max_positions: int, max_seq_per_call: int,
                  max_tokens_per_call: int, page_size: int = 16, rope_base: float = 10000.0,
+                 policy: str = "unit", sink: int = 0, recent: int = 0,
                  device: str = "cuda", stream=None):
         import torch
         self.lib = load_library()
         self.cfg = Config(n_sessions, layers, q_heads, kv_heads, head_dim, page_size, budget,
                           window, KVC_BF16 if dtype == "bf16" else KVC_F32, rope_base, n_pages,
                           max_pages_per_session, max_positions, max_seq_per_call,
-                          max_tokens_per_call)
+                          max_tokens_per_call, POLICIES[policy], sink, recent)
         self.dtype = dtype
         self.torch_dtype = torch.bfloat16 if dtype == "bf16" else torch.float32
         pool_bytes, meta_bytes = query_sizes(self.cfg)

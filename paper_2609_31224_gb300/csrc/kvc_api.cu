@@ -131,6 +131,10 @@ int check_config(const kvc_config* c) {
   if (!((c->dtype == KVC_BF16 && c->head_dim == 128) || (c->dtype == KVC_F32 && c->head_dim == 64)))
     return fail(KVC_EINVAL, "supported (dtype, head_dim): (KVC_BF16, 128), (KVC_F32, 64)");
   if (c->window < 0) return fail(KVC_EINVAL, "window must be >= 0");
+  if (c->policy < KVC_POLICY_UNIT || c->policy > KVC_POLICY_SINK_RECENT)
+    return fail(KVC_EINVAL, "policy must be one of KVC_POLICY_UNIT, _POSITION, _SINK_RECENT");
+  if (c->policy == KVC_POLICY_SINK_RECENT && (c->sink < 0 || c->recent < 0))
+    return fail(KVC_EINVAL, "sink and recent must be >= 0");
   if (!(c->rope_base > 0.0)) return fail(KVC_EINVAL, "rope_base must be > 0");
   if (c->n_pages < 1) return fail(KVC_EINVAL, "n_pages must be >= 1");
   const int64_t rows = c->n_pages * c->layers * 2 * c->kv_heads * PS;
@@ -252,6 +256,9 @@ int kvc_create(kvc_ctx** out, const kvc_config* cfg, void* d_pool, size_t pool_b
   d.max_tokens = cfg->max_tokens_per_call;
   d.budget = cfg->budget;
   d.window = cfg->window;
+  d.policy = cfg->policy;
+  d.sink = cfg->sink;
+  d.recent = cfg->recent;
   d.n_pages = cfg->n_pages;
   d.pool = static_cast<uint8_t*>(d_pool);
   layout_meta(*cfg, static_cast<uint8_t*>(d_meta), &d);

@@ -81,6 +81,7 @@ struct Dev {
   int32_t max_pages_per_session, max_positions, max_seq, max_tokens;
   int64_t budget;
   int32_t window;
+  int32_t policy, sink, recent;  // KVC_POLICY_*
   int64_t n_pages;
   int32_t bitmap_words;
   int32_t max_moves;

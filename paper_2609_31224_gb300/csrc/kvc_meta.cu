@@ -373,7 +373,7 @@ __global__ void __launch_bounds__(256) append_kv_kernel(Dev d, int total, const 
 // freeing of consumed live pages, state update.
 // ---------------------------------------------------------------------------
 struct LiveSlot {
-  int unit, type, gs;
+  int unit, type, gs, pos;
 };
 
 __device__ inline LiveSlot live_slot(const Dev& d, const SessState& st, const int32_t* row,
@@ -384,7 +384,60 @@ __device__ inline LiveSlot live_slot(const Dev& d, const SessState& st, const in
   r.gs = gs;
   r.unit = d.meta_unit[gs];
   r.type = d.meta_type[gs];
+  r.pos = d.meta_pos[gs];
   return r;
+}
+
+// Whether a slot inside the consumed live prefix is dropped: its type under the
+// rule of Sec. 3.3 and its position-granular variant; its position under the
+// sink + recent variant.
+__device__ inline bool slot_evicted(const Dev& d, const LiveSlot& ls) {
+  if (d.policy == KVC_POLICY_SINK_RECENT) return ls.pos >= d.sink;
+  return ls.unit >= 0 && evictable_type(ls.type);
+}
+
+// Length of the live prefix a position-granular evict consumes: up to and
+// including the need-th evictable slot of a unit <= lim (fewer if fewer exist;
+// those units are a prefix of the live region).  One warp.
+__device__ int position_variant_end(const Dev& d, const SessState& st, const int32_t* row,
+                                    int lim, int need, int lane) {
+  int cnt = 0, end = 0;
+  for (int w0 = 0; w0 < st.n_live; w0 += 32) {
+    const int j = w0 + lane;
+    const bool valid = j < st.n_live;
+    LiveSlot ls = {INT_MAX, 0, 0, 0};
+    if (valid) ls = live_slot(d, st, row, j);
+    const unsigned stop = __ballot_sync(FULL, !valid || ls.unit > lim);
+    const int first_stop = stop ? __ffs(stop) - 1 : 32;
+    const unsigned ev = __ballot_sync(FULL, lane < first_stop && ls.unit >= 0 &&
+                                                evictable_type(ls.type));
+    const int n_ev = __popc(ev);
+    if (cnt + n_ev >= need) {
+      unsigned m = ev;  // drop the (need - cnt - 1) lowest set bits: the next is the need-th
+      for (int k = need - cnt - 1; k > 0; --k) m &= m - 1;
+      return w0 + (__ffs(m) - 1) + 1;
+    }
+    if (ev) end = w0 + (31 - __clz(ev)) + 1;
+    cnt += n_ev;
+    if (stop) break;
+  }
+  return end;
+}
+
+// Length of the live prefix a sink + recent evict consumes: every live slot
+// whose position is below pos_next - recent (positions ascend along the region).
+__device__ int sink_recent_end(const Dev& d, const SessState& st, const int32_t* row,
+                               int lane) {
+  const int hi = st.pos_next - d.recent;
+  int end = 0;
+  for (int w0 = 0; w0 < st.n_live; w0 += 32) {
+    const int j = w0 + lane;
+    const bool in = j < st.n_live && live_slot(d, st, row, j).pos < hi;
+    const unsigned b = __ballot_sync(FULL, in);
+    end += __popc(b);
+    if (b != FULL) break;
+  }
+  return end;
 }
 
 __global__ void __launch_bounds__(META_THREADS) evict_plan_kernel(Dev d, SeqArgs a,
@@ -408,14 +461,15 @@ __global__ void __launch_bounds__(META_THREADS) evict_plan_kernel(Dev d, SeqArgs
     const int r0 = st.n_hist + st.n_live;
     const int lim = st.unit_cur - d.window;
     int ustar = -2;
-    if (d.budget >= 0 && (int64_t)r0 > d.budget && st.n_live > 0) {
+    if (d.policy == KVC_POLICY_UNIT && d.budget >= 0 && (int64_t)r0 > d.budget &&
+        st.n_live > 0) {
       int e_before = 0;        // evictable slots before this window
       int prev_unit = INT_MIN; // unit of the slot just before this window
       int e_at_prev_start = 0; // evictable count before prev_unit's first slot
       for (int w0 = 0; w0 < st.n_live; w0 += 32) {
         const int j = w0 + lane;
         const bool valid = j < st.n_live;
-        LiveSlot ls = {INT_MAX, 0, 0};
+        LiveSlot ls = {INT_MAX, 0, 0, 0};
         if (valid) ls = live_slot(d, st, row, j);
         const bool ev = valid && ls.unit >= 0 && evictable_type(ls.type);
         const unsigned bal_ev = __ballot_sync(FULL, ev);
@@ -442,15 +496,25 @@ __global__ void __launch_bounds__(META_THREADS) evict_plan_kernel(Dev d, SeqArgs
         e_before += __popc(bal_ev);
       }
     }
+    // The consumed live prefix: units <= u* under the rule; for the variants its
+    // length is decided first.
     int end = 0, surv = 0, nev = 0;
-    if (ustar >= 0) {
+    int vend = -1;
+    if (d.policy == KVC_POLICY_POSITION) {
+      vend = (d.budget >= 0 && (int64_t)r0 > d.budget)
+                 ? position_variant_end(d, st, row, lim, (int)(r0 - d.budget), lane)
+                 : 0;
+    } else if (d.policy == KVC_POLICY_SINK_RECENT) {
+      vend = sink_recent_end(d, st, row, lane);
+    }
+    if (ustar >= 0 || vend > 0) {
       for (int w0 = 0; w0 < st.n_live; w0 += 32) {
         const int j = w0 + lane;
         const bool valid = j < st.n_live;
-        LiveSlot ls = {INT_MAX, 0, 0};
+        LiveSlot ls = {INT_MAX, 0, 0, 0};
         if (valid) ls = live_slot(d, st, row, j);
-        const bool in = valid && ls.unit <= ustar;
-        const bool ev = in && ls.unit >= 0 && evictable_type(ls.type);
+        const bool in = valid && (vend >= 0 ? j < vend : ls.unit <= ustar);
+        const bool ev = in && slot_evicted(d, ls);
         const unsigned bin = __ballot_sync(FULL, in);
         end += __popc(bin);
         nev += __popc(__ballot_sync(FULL, ev));
@@ -517,9 +581,9 @@ __global__ void __launch_bounds__(META_THREADS) evict_plan_kernel(Dev d, SeqArgs
     for (int w0 = 0; w0 < end; w0 += 32) {
       const int j = w0 + lane;
       const bool in = j < end;
-      LiveSlot ls = {0, 0, 0};
+      LiveSlot ls = {0, 0, 0, 0};
       if (in) ls = live_slot(d, st, lrow, j);
-      const bool sv = in && !(ls.unit >= 0 && evictable_type(ls.type));
+      const bool sv = in && !slot_evicted(d, ls);
       const unsigned bal = __ballot_sync(FULL, sv);
       if (sv) {
         const int k = done + __popc(bal & lanemask_lt());

@@ -92,7 +92,8 @@ class Driver:
                                       q_heads=w.q_heads, kv_heads=w.kv_heads,
                                       head_dim=w.head_dim, budget=w.budget, window=w.window,
                                       dtype=w.dtype, rope_base=w.rope_base,
-                                      page_size=w.page_size, device=device, **self.sizing)
+                                      page_size=w.page_size, policy=w.policy, sink=w.sink,
+                                      recent=w.recent, device=device, **self.sizing)
         self.pos = np.zeros(w.n_sessions, dtype=np.int64)  # host copy of positions fed
         self.tdtype = torch.bfloat16 if w.dtype == "bf16" else torch.float32
         self.step_index = 0

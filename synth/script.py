@@ -57,6 +57,9 @@ class Workload:
     q_scale: float = 1.0
     kv_scale: float = 1.0
     rope_base: float = 10000.0
+    policy: str = "unit"         # eviction policy: "unit" (Sec. 3.3), "position", "sink_recent"
+    sink: int = 0                # sink_recent: first positions kept
+    recent: int = 0              # sink_recent: most recent positions kept
 
     @property
     def group(self) -> int:

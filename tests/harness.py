@@ -41,7 +41,8 @@ class Lockstep:
         self.orc = OracleCache(OracleConfig(
             n_sessions=w.n_sessions, layers=w.layers, q_heads=w.q_heads, kv_heads=w.kv_heads,
             head_dim=w.head_dim, page_size=w.page_size, budget=w.budget, window=w.window,
-            dtype=w.dtype, rope_base=w.rope_base, n_pages=driver.sizing["n_pages"]))
+            dtype=w.dtype, rope_base=w.rope_base, n_pages=driver.sizing["n_pages"],
+            policy=w.policy, sink=w.sink, recent=w.recent))
         self.stats = []
         self.n_compared = 0
 

@@ -90,6 +90,43 @@ def test_small_bf16_mixed_segments(budget, window, seed):
     assert ls.n_compared > 100
 
 
+@pytest.mark.parametrize("policy,budget,window,sink,recent", [
+    ("position", 64, 2, 0, 0), ("position", 0, 0, 0, 0), ("position", 100, 5, 0, 0),
+    ("sink_recent", 64, 0, 4, 40), ("sink_recent", 64, 0, 0, 7), ("sink_recent", 64, 0, 37, 0)])
+def test_policy_variants_small_bf16(policy, budget, window, sink, recent):
+    """The position-granular and sink + recent variants of the eviction step on the
+    same kernels: every state bit-exact after every evict, every output compared."""
+    w = S.SINGLE_BF16.with_(layers=2, n_sessions=3, budget=budget, window=window, seed=21,
+                            turn_period=10, turn_jitter=1, policy=policy, sink=sink,
+                            recent=recent)
+    ls, _ = _lockstep(w, n_units=40)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda *a: True)
+    assert ls.n_compared > 0
+    assert any(ls.drv.cache.export_state(s)["n_evicted"] > 0 for s in range(3))
+
+
+@pytest.mark.parametrize("policy", ["position", "sink_recent"])
+def test_policy_variants_tiny_f32(policy):
+    w = S.TINY_F32.with_(policy=policy, sink=4, recent=300)
+    ls, _ = _lockstep(w)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda *a: True)
+    assert ls.drv.cache.export_state(0)["n_evicted"] > 0
+
+
+def test_position_variant_single_session_full_size():
+    """The position-granular variant on the full-size single-session workload: every evict
+    bit-exact (the resident count lands on B exactly), attention sampled."""
+    ls, _ = _lockstep(S.SINGLE_BF16.with_(policy="position"))
+    samples = {190, 420, 599}
+    for step in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda st, kind, i, layer: st in samples and layer in (0, 31)
+                    and i in (0, 1))
+    st = ls.drv.cache.export_state(0)
+    assert st["resident"] == 4096
+
+
 def test_sharp_attention_bf16():
     """Larger query scale makes the softmax peaked, so a wrong key order shows.
 
