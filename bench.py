@@ -413,6 +413,50 @@ def run_unbounded_comparison() -> dict:
             "attention_time_ratio_full_over_budget": f["attention_ms"] / b["attention_ms"]}
 
 
+# -- Table-3-shaped budget sweep ---------------------------------------------------------------
+def run_budget_sweep(n_sessions: int) -> dict:
+    """Budgets B in {unbounded, 8K, 6K, 4K, 0 (floor)} on full-size single sessions (32
+    layers, 600 units, batch size 1, one session at a time): End and Peak resident
+    positions (means over sessions) and the path's GPU time per unit (append, every
+    layer's attention and the evict of one unit; CUDA events), mean and p99."""
+    import numpy as np
+    import torch
+    from synth import script as S
+    from synth.driver import Driver
+    rows = []
+    for budget in (-1, 8192, 6144, 4096, 0):
+        w = S.SINGLE_BF16.with_(name=f"single-bf16-32L-600u-B{budget}-W10", budget=budget,
+                                n_sessions=n_sessions)
+        ends, peaks, unit_ms = [], [], []
+        for sid in range(n_sessions):
+            drv = Driver(w, [S.session_script(w, sid)])
+            spans = []
+            for _ in range(len(drv.sched)):
+                st = drv.prepare_step()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                drv.run_step(st)
+                e1.record()
+                spans.append((e0, e1))
+                del st
+            torch.cuda.synchronize()
+            unit_ms += [a.elapsed_time(b) for a, b in spans]
+            info = drv.cache.export_state(sid)
+            ends.append(info["resident"])
+            peaks.append(info["peak_resident"])
+            del drv
+            torch.cuda.empty_cache()
+        t = np.array(unit_ms)
+        rows.append({"budget": "unbounded" if budget < 0 else budget,
+                     "end_positions": float(np.mean(ends)), "peak_positions": float(np.mean(peaks)),
+                     "unit_ms_mean": float(t.mean()), "unit_ms_p99": float(np.percentile(t, 99)),
+                     "units": int(t.size)})
+    return {"sweep": "Table-3-shaped budget sweep, synthetic single-session workload "
+                     "(32 layers, 32/8 heads, D=128, bf16, W=10, 600 units, batch size 1)",
+            "sessions_per_budget": n_sessions, "rows": rows}
+
+
 # -- the oracle on the host cores -----------------------------------------------------------------
 def oracle_sample(layers_sampled: int = 1, session: int = 0, start: int | None = None) -> dict:
     """Time the CPU oracle on one session's unit at the benchmark's steady state, for
@@ -499,6 +543,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--compare-unbounded", action="store_true",
                     help="print the B=4096 vs B=infinity single-session comparison and exit")
+    ap.add_argument("--budget-sweep", type=int, default=0, metavar="SESSIONS",
+                    help="print the Table-3-shaped budget sweep over SESSIONS sessions and exit")
     ap.add_argument("--sessions", type=int, default=None,
                     help="reduced case for profiler captures (default: the full 64)")
     ap.add_argument("--layers", type=int, default=None,
@@ -526,6 +572,10 @@ def main():
     if args.compare_unbounded:
         if rank == 0:
             print(json.dumps(run_unbounded_comparison()))
+        return
+    if args.budget_sweep:
+        if rank == 0:
+            print(json.dumps(run_budget_sweep(args.budget_sweep)))
         return
     out = run_ours(args, rank, world, local_rank)
     if rank == 0:
