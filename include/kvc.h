@@ -229,6 +229,23 @@ int kvc_export_state(kvc_ctx* ctx, int session, kvc_session_info* h_info,
  * order, to host buffers [cap][Hkv][D] each (synchronises). */
 int kvc_export_kv(kvc_ctx* ctx, int session, int layer, void* h_k, void* h_v, int64_t cap);
 
+/* Transcript export for query-time re-encoding (Sec. 4.2: task queries use
+ * only the incoming-speech transcript, re-encoded after the streaming cache is
+ * discarded).  Gathers one session's retained TRANSCRIPT positions, in position
+ * order, with their stored K (rotated at the original position) and V of every
+ * layer.  Asynchronous on stream; uses the eviction move list as scratch (stream
+ * order keeps it apart from kvc_evict).  Leaves the cache unchanged.
+ *   session    0 .. n_sessions-1
+ *   cap        capacity in positions of the outputs; 0 <= cap <= the move list's
+ *              capacity (max_seq_per_call * max_pages_per_session * page_size)
+ *   d_pos_out  device [cap] int32: original positions
+ *   d_k_out, d_v_out  device [L][cap][Hkv][D] each, the cache's element type,
+ *              16-byte aligned
+ *   d_count    device int32: number of TRANSCRIPT positions retained; the first
+ *              min(count, cap) of them are written */
+int kvc_export_transcript(kvc_ctx* ctx, int session, int64_t cap, int32_t* d_pos_out,
+                          void* d_k_out, void* d_v_out, int32_t* d_count, void* stream);
+
 /* Free pages in the pool and the device error word (synchronises). */
 int kvc_device_status(kvc_ctx* ctx, int64_t* h_free_pages, int32_t* h_error_bits);
 

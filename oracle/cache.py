@@ -17,6 +17,7 @@ from .layout import PagePool, SessionLayout
 from .numerics import round_storage
 from .policy import SessionPolicy
 from .rope import rope
+from synth.script import TRANSCRIPT
 
 
 @dataclass
@@ -85,6 +86,12 @@ class OracleCache:
             self.policy[s] = SessionPolicy(self.cfg.budget, self.cfg.window)
             self.layout[s] = SessionLayout(self.cfg.page_size)
         self.last_append = None
+
+    def transcript_positions(self, s: int) -> list[int]:
+        """Retained TRANSCRIPT positions in retained order (what query-time re-encoding
+        reads after the streaming cache is discarded, Sec. 4.2)."""
+        pol = self.policy[s]
+        return [p for p in pol.retained_positions() if pol.type[p] == TRANSCRIPT]
 
     def resident_size(self, s: int) -> int:
         return self.policy[s].resident()

@@ -27,7 +27,8 @@ STATUS = {0: "KVC_OK", -1: "KVC_EINVAL", -2: "KVC_ENOMEM", -3: "KVC_ECUDA", -4: 
 EXPORTED = ["kvc_query_sizes", "kvc_create", "kvc_destroy", "kvc_append_chunk", "kvc_evict",
             "kvc_attn_prefill_chunk", "kvc_attn_decode", "kvc_attn_decode_noalloc",
             "kvc_resident_size", "kvc_release",
-            "kvc_export_state", "kvc_export_kv", "kvc_device_status", "kvc_last_error"]
+            "kvc_export_state", "kvc_export_kv", "kvc_export_transcript", "kvc_device_status",
+            "kvc_last_error"]
 
 
 class KvcError(RuntimeError):
@@ -83,6 +84,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.kvc_export_state.argtypes = [vp, ctypes.c_int, ctypes.POINTER(SessionInfo), p_i32, p_i32,
                                      p_i32, ctypes.POINTER(ctypes.c_uint8), p_i32, i64]
     lib.kvc_export_kv.argtypes = [vp, ctypes.c_int, ctypes.c_int, vp, vp, i64]
+    lib.kvc_export_transcript.argtypes = [vp, ctypes.c_int, i64, vp, vp, vp, vp, vp]
     lib.kvc_device_status.argtypes = [vp, ctypes.POINTER(i64), ctypes.POINTER(i32)]
     lib.kvc_last_error.restype = ctypes.c_char_p
     for name in EXPORTED:
@@ -250,6 +252,21 @@ class KVCache:
             k = (k.astype(np.uint32) << 16).view(np.float32)
             v = (v.astype(np.uint32) << 16).view(np.float32)
         return k[:n], v[:n]
+
+    def export_transcript(self, session: int, cap: int, stream=None):
+        """Retained TRANSCRIPT positions of a session (Sec. 4.2), with their stored K and V
+        of every layer: device tensors (positions [cap] int32, K and V [L][cap][Hkv][D],
+        count [1] int32), filled asynchronously on the stream."""
+        import torch
+        dev = self.pool.device
+        shape = (self.cfg.layers, max(1, cap), self.cfg.kv_heads, self.cfg.head_dim)
+        pos = torch.zeros(max(1, cap), dtype=torch.int32, device=dev)
+        k = torch.zeros(shape, dtype=self.torch_dtype, device=dev)
+        v = torch.zeros(shape, dtype=self.torch_dtype, device=dev)
+        count = torch.zeros(1, dtype=torch.int32, device=dev)
+        _check(self.lib.kvc_export_transcript(self.ctx, session, cap, pos.data_ptr(), k.data_ptr(),
+                                              v.data_ptr(), count.data_ptr(), _stream(stream)))
+        return pos, k, v, count
 
     def device_status(self) -> tuple[int, int]:
         free, err = ctypes.c_int64(), ctypes.c_int32()

@@ -522,6 +522,23 @@ int kvc_export_state(kvc_ctx* ctx, int session, kvc_session_info* h_info, int32_
   return KVC_OK;
 }
 
+int kvc_export_transcript(kvc_ctx* ctx, int session, int64_t cap, int32_t* d_pos_out,
+                          void* d_k_out, void* d_v_out, int32_t* d_count, void* stream) {
+  g_err.clear();
+  if (!ctx || !d_count) return fail(KVC_EINVAL, "ctx / d_count is NULL");
+  if (session < 0 || session >= ctx->cfg.n_sessions)
+    return fail(KVC_EINVAL, "session id %d out of range", session);
+  if (cap < 0 || cap > ctx->d.max_moves)
+    return fail(KVC_EINVAL, "cap must be in 0..%d", ctx->d.max_moves);
+  if (cap > 0 && (!d_pos_out || !d_k_out || !d_v_out))
+    return fail(KVC_EINVAL, "output buffers are NULL");
+  if (cap > 0 && (!aligned16(d_k_out) || !aligned16(d_v_out)))
+    return fail(KVC_EINVAL, "d_k_out / d_v_out must be 16-byte aligned");
+  KVC_CUDA(launch_transcript(ctx->d, session, (int)cap, d_pos_out, d_k_out, d_v_out, d_count,
+                             static_cast<cudaStream_t>(stream)));
+  return KVC_OK;
+}
+
 int kvc_export_kv(kvc_ctx* ctx, int session, int layer, void* h_k, void* h_v, int64_t cap) {
   g_err.clear();
   if (!ctx || !h_k || !h_v) return fail(KVC_EINVAL, "ctx / h_k / h_v is NULL");

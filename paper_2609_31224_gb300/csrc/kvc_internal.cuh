@@ -400,6 +400,8 @@ cudaError_t launch_append(const Dev& d, const AppendArgs& a, const uint8_t* type
                           const void* v, cudaStream_t s);
 cudaError_t launch_evict(const Dev& d, const SeqArgs& a, int64_t* resident_out, cudaStream_t s);
 cudaError_t launch_release(const Dev& d, const SeqArgs& a, cudaStream_t s);
+cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_out, void* k_out,
+                              void* v_out, int32_t* count, cudaStream_t s);
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                bool pdl, cudaStream_t s);
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,

@@ -660,6 +660,74 @@ __global__ void __launch_bounds__(256) evict_copy_kernel(Dev d) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// Transcript export (Sec. 4.2): one session's retained TRANSCRIPT positions in
+// retained (= position) order.  Part 1 (one CTA): compaction of the retained
+// slots by type (block scan); the global slots go to the move list, used as
+// scratch, and the positions to pos_out.  Part 2: K and V rows of every layer.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(META_THREADS) transcript_gather_kernel(Dev d, int sid, int cap,
+                                                                         int32_t* pos_out,
+                                                                         int32_t* count) {
+  __shared__ int s_warp[33];
+  const SessState st = d.sess[sid];
+  const int n = st.n_hist + st.n_live;
+  const int32_t* hrow = d.hist_pt + (size_t)sid * d.max_pages_per_session;
+  const int32_t* lrow = d.live_pt + (size_t)sid * d.max_pages_per_session;
+  int done = 0;
+  for (int b0 = 0; b0 < n; b0 += META_THREADS) {
+    const int i = b0 + threadIdx.x;
+    int gs = 0;
+    bool tr = false;
+    if (i < n) {
+      if (i < st.n_hist) {
+        gs = hrow[i / PS] * PS + i % PS;
+      } else {
+        const int j = st.live_head + i - st.n_hist;
+        gs = lrow[j / PS] * PS + j % PS;
+      }
+      tr = d.meta_type[gs] == KVC_TRANSCRIPT;
+    }
+    int total;
+    const int idx = done + block_exclusive_scan(tr ? 1 : 0, &total, s_warp);
+    if (tr && idx < cap) {
+      pos_out[idx] = d.meta_pos[gs];
+      d.moves[idx] = make_int2(gs, 0);
+    }
+    done += total;
+    __syncthreads();  // s_warp is reused by the next scan
+  }
+  if (threadIdx.x == 0) {
+    *count = done;
+    d.g->n_moves = min(done, cap);
+  }
+}
+
+// Rows [L][cap][Hkv][D] of K and V; 16-byte units, grid-stride.
+__global__ void __launch_bounds__(256) transcript_copy_kernel(Dev d, int cap, uint8_t* k_out,
+                                                              uint8_t* v_out) {
+  const int n = d.g->n_moves;
+  const int vec_per_row = d.head_dim * d.esz / 16;
+  const int64_t total = (int64_t)n * d.layers * 2 * d.kv_heads * vec_per_row;
+  for (int64_t u = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; u < total;
+       u += (int64_t)gridDim.x * blockDim.x) {
+    const int v = (int)(u % vec_per_row);
+    int64_t r = u / vec_per_row;
+    const int h = (int)(r % d.kv_heads);
+    r /= d.kv_heads;
+    const int kv = (int)(r % 2);
+    r /= 2;
+    const int i = (int)(r % n);
+    const int l = (int)(r / n);
+    const int gs = d.moves[i].x;
+    const size_t src = pool_offset_elems(d, gs / PS, l, kv, h, gs % PS) * d.esz + (size_t)v * 16;
+    const size_t dst =
+        (((size_t)l * cap + i) * d.kv_heads + h) * d.head_dim * d.esz + (size_t)v * 16;
+    *reinterpret_cast<uint4*>((kv ? v_out : k_out) + dst) =
+        *reinterpret_cast<const uint4*>(d.pool + src);
+  }
+}
+
 // Release (one CTA): free every page of the listed sessions and reset them.
 __global__ void __launch_bounds__(META_THREADS) release_kernel(Dev d, SeqArgs a) {
   __shared__ int s_freed;
@@ -719,6 +787,17 @@ cudaError_t launch_evict(const Dev& d, const SeqArgs& a, int64_t* resident_out, 
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   evict_copy_kernel<<<sms * 4, 256, 0, s>>>(d);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_out, void* k_out,
+                              void* v_out, int32_t* count, cudaStream_t s) {
+  transcript_gather_kernel<<<1, META_THREADS, 0, s>>>(d, session, cap, pos_out, count);
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  transcript_copy_kernel<<<sms * 4, 256, 0, s>>>(d, cap, static_cast<uint8_t*>(k_out),
+                                                 static_cast<uint8_t*>(v_out));
   return cudaGetLastError();
 }
 

@@ -127,6 +127,36 @@ def test_position_variant_single_session_full_size():
     assert st["resident"] == 4096
 
 
+def test_transcript_export():
+    """Transcript export (Sec. 4.2): positions bit-exact against the oracle, K and V
+    bit-exact against the stored rows of those positions, count exact, and a short
+    capacity keeps the first positions."""
+    w = S.SINGLE_BF16.with_(layers=2, n_sessions=3, budget=64, window=2, seed=5,
+                            p_no_segment=0.1, p_long_segment=0.1, turn_period=12, turn_jitter=2)
+    ls, _ = _lockstep(w, n_units=40)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=None)
+    cache = ls.drv.cache
+    for s in range(3):
+        want = ls.orc.transcript_positions(s)
+        st = cache.export_state(s)
+        pos, k, v, count = cache.export_transcript(s, st["resident"])
+        torch.cuda.synchronize()
+        n = int(count.item())
+        assert n == len(want) > 0
+        assert pos[:n].cpu().numpy().tolist() == want
+        idx = [st["pos"].index(p) for p in want]
+        for layer in range(w.layers):
+            ks, vs = cache.export_kv(s, layer)
+            assert np.array_equal(k[layer, :n].float().cpu().numpy(), ks[idx])
+            assert np.array_equal(v[layer, :n].float().cpu().numpy(), vs[idx])
+        pos2, k2, _, count2 = cache.export_transcript(s, 3)
+        torch.cuda.synchronize()
+        assert int(count2.item()) == n
+        assert pos2.cpu().numpy().tolist() == want[:3]
+        assert torch.equal(k2[:, :3], k[:, :3])
+
+
 def test_sharp_attention_bf16():
     """Larger query scale makes the softmax peaked, so a wrong key order shows.
 

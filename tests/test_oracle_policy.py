@@ -409,3 +409,26 @@ def test_layout_invariants_policy_variants(policy, seed):
                 seen.add(pid)
             used += len(lay.hist_pages) + len(lay.live_pages)
         assert used + c.pool.free_count() == total
+
+
+@pytest.mark.parametrize("policy", ["unit", "position"])
+def test_transcript_export_keeps_every_transcript(policy):
+    """Transcripts are never evicted by the rule (or its position-granular reading), so the
+    transcript record after any number of evicts is every TRANSCRIPT position fed."""
+    rng = np.random.default_rng(11)
+    c = _cache(40, 1, n_sessions=2)
+    c.policy = [SessionPolicy(40, 1, policy=policy) for _ in range(2)]
+    fed = {0: [], 1: []}
+    for _ in range(30):
+        chunks = []
+        for s in (0, 1):
+            unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * int(rng.integers(0, 9)) + [ASR_DELIM] + \
+                [TRANSCRIPT] * int(rng.poisson(2)) + [ASR_DELIM] + [TEXT] * int(rng.integers(0, 3))
+            base = c.policy[s].pos_next
+            fed[s] += [base + i for i, t in enumerate(unit) if t == TRANSCRIPT]
+            chunks.append(unit)
+        c.append_chunk([0, 1], chunks)
+        c.evict([0, 1])
+    for s in (0, 1):
+        assert c.transcript_positions(s) == fed[s]
+        assert any(c.policy[s].evicted)
