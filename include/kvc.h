@@ -146,12 +146,23 @@ void kvc_destroy(kvc_ctx* ctx);
  *   h_cu_tokens  host [n_seq+1] token offsets, h_cu_tokens[0] = 0, every
  *                session gets >= 1 token; total <= max_tokens_per_call
  *   d_types      device [total] type bytes
- *   d_k, d_v     device [L][total][Hkv][D] un-rotated keys / values
+ *   d_k, d_v     device [L][total][Hkv][D] un-rotated keys / values, or both NULL
+ *                to write the layers one by one with kvc_append_kv_layer
  * Returns KVC_ENOMEM (nothing launched) if the pool cannot hold the chunk.
  * The chunk's queries are what the following attention calls answer. */
 int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions,
                      const int32_t* h_cu_tokens, const uint8_t* d_types, const void* d_k,
                      const void* d_v, void* stream);
+
+/* Per-layer K/V of the last append, for the model's real order (layer l's K/V
+ * exist only after layer l's projections): call kvc_append_chunk with d_k =
+ * d_v = NULL (positions, units, pages and tags only), then this for each layer
+ * before that layer's attention.  Writes K rotated at its position and V into
+ * the chunk's slots.  Attention on a layer whose K/V are not written returns
+ * KVC_ESTATE.
+ *   layer      0 .. L-1
+ *   d_k, d_v   device [total][Hkv][D], total and order as in the last append */
+int kvc_append_kv_layer(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v, void* stream);
 
 /* Online eviction (Sec. 3.3) for each listed session, run by the caller after
  * a unit: while resident > B, evict the ACOUSTIC and ASR_DELIM positions of

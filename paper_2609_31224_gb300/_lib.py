@@ -24,7 +24,8 @@ POLICIES = {"unit": KVC_POLICY_UNIT, "position": KVC_POLICY_POSITION,
 STATUS = {0: "KVC_OK", -1: "KVC_EINVAL", -2: "KVC_ENOMEM", -3: "KVC_ECUDA", -4: "KVC_ESTATE",
           -5: "KVC_EDEVICE"}
 
-EXPORTED = ["kvc_query_sizes", "kvc_create", "kvc_destroy", "kvc_append_chunk", "kvc_evict",
+EXPORTED = ["kvc_query_sizes", "kvc_create", "kvc_destroy", "kvc_append_chunk",
+            "kvc_append_kv_layer", "kvc_evict",
             "kvc_attn_prefill_chunk", "kvc_attn_decode", "kvc_attn_decode_noalloc",
             "kvc_resident_size", "kvc_release",
             "kvc_export_state", "kvc_export_kv", "kvc_export_transcript", "kvc_device_status",
@@ -75,6 +76,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.kvc_destroy.argtypes = [vp]
     lib.kvc_destroy.restype = None
     lib.kvc_append_chunk.argtypes = [vp, ctypes.c_int, p_i32, p_i32, vp, vp, vp, vp]
+    lib.kvc_append_kv_layer.argtypes = [vp, ctypes.c_int, vp, vp, vp]
     lib.kvc_evict.argtypes = [vp, ctypes.c_int, p_i32, vp, vp]
     lib.kvc_attn_prefill_chunk.argtypes = [vp, ctypes.c_int, vp, vp, vp]
     lib.kvc_attn_decode.argtypes = [vp, ctypes.c_int, vp, vp, vp]
@@ -189,8 +191,18 @@ class KVCache:
     def append_chunk(self, sessions, cu_tokens, types, k, v, stream=None) -> None:
         s, cu = _i32(sessions), _i32(cu_tokens)
         _check(self.lib.kvc_append_chunk(self.ctx, len(s), _ptr_i32(s), _ptr_i32(cu),
-                                         types.data_ptr(), k.data_ptr(), v.data_ptr(),
-                                         _stream(stream)))
+                                         types.data_ptr(), None if k is None else k.data_ptr(),
+                                         None if v is None else v.data_ptr(), _stream(stream)))
+
+    def append_kv_layer(self, layer: int, k, v, stream=None) -> None:
+        """One layer's K/V [total][Hkv][D] of the last append (after an append without K/V)."""
+        _check(self.lib.kvc_append_kv_layer(self.ctx, layer, k.data_ptr(), v.data_ptr(),
+                                            _stream(stream)))
+
+    def append_kv_layer_raw(self, layer, k_ptr, v_ptr, stream) -> None:
+        rc = self.lib.kvc_append_kv_layer(self.ctx, layer, k_ptr, v_ptr, stream)
+        if rc:
+            _check(rc)
 
     def evict(self, sessions, resident_out=None, stream=None) -> None:
         s = _i32(sessions)

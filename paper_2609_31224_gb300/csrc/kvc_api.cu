@@ -167,7 +167,8 @@ struct kvc_ctx {
   // Last append (queries of the following attention calls).
   bool attn_valid = false;
   int last_n_seq = 0, last_total = 0, last_max_t = 0;
-  int attn_since_append = 0;  // attention launches since the last append
+  int attn_since_append = 0;  // attention launches since the last append (or layer write)
+  uint64_t layers_written = 0;  // layers whose K/V of the last append are in the pool
   bool last_single = false;
   int pf_target = 0;
 };
@@ -297,8 +298,11 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, const i
   int rc = check_sessions(ctx, n_seq, h_sessions);
   if (rc) return rc;
   if (!h_cu_tokens) return fail(KVC_EINVAL, "h_cu_tokens is NULL");
-  if (!d_types || !d_k || !d_v) return fail(KVC_EINVAL, "d_types / d_k / d_v must be non-NULL");
-  if (!aligned16(d_k) || !aligned16(d_v)) return fail(KVC_EINVAL, "d_k / d_v must be 16-byte aligned");
+  if (!d_types) return fail(KVC_EINVAL, "d_types must be non-NULL");
+  if ((d_k == nullptr) != (d_v == nullptr))
+    return fail(KVC_EINVAL, "d_k and d_v must both be given or both be NULL");
+  if (d_k && (!aligned16(d_k) || !aligned16(d_v)))
+    return fail(KVC_EINVAL, "d_k / d_v must be 16-byte aligned");
   if (h_cu_tokens[0] != 0) return fail(KVC_EINVAL, "h_cu_tokens[0] must be 0");
   int64_t need = 0;
   int max_t = 0;
@@ -346,10 +350,29 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, const i
   ctx->delta_since_readback += need;
   ctx->attn_valid = true;
   ctx->attn_since_append = 0;
+  ctx->layers_written = d_k ? (ctx->cfg.layers == 64 ? ~0ull : (1ull << ctx->cfg.layers) - 1) : 0;
   ctx->last_n_seq = n_seq;
   ctx->last_total = total;
   ctx->last_max_t = max_t;
   ctx->last_single = single;
+  return KVC_OK;
+}
+
+int kvc_append_kv_layer(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v, void* stream) {
+  g_err.clear();
+  if (!ctx) return fail(KVC_EINVAL, "ctx is NULL");
+  if (layer < 0 || layer >= ctx->cfg.layers)
+    return fail(KVC_EINVAL, "layer %d outside 0..%d", layer, ctx->cfg.layers - 1);
+  if (!d_k || !d_v) return fail(KVC_EINVAL, "d_k / d_v must be non-NULL");
+  if (!aligned16(d_k) || !aligned16(d_v)) return fail(KVC_EINVAL, "d_k / d_v must be 16-byte aligned");
+  if (!ctx->attn_valid)
+    return fail(KVC_ESTATE, "kvc_append_kv_layer needs a preceding kvc_append_chunk (no evict/release after it)");
+  KVC_CUDA(launch_append_layers(ctx->d, ctx->last_total, layer, 1, d_k, d_v,
+                                static_cast<cudaStream_t>(stream)));
+  ctx->layers_written |= 1ull << layer;
+  // The next attention launch must not start early: its prologue loads pages
+  // this write may still be filling.
+  ctx->attn_since_append = 0;
   return KVC_OK;
 }
 
@@ -397,6 +420,9 @@ static int check_attn(kvc_ctx* ctx, int layer, const void* d_q, void* d_out) {
   if (!aligned16(d_q) || !aligned16(d_out)) return fail(KVC_EINVAL, "d_q / d_out must be 16-byte aligned");
   if (!ctx->attn_valid)
     return fail(KVC_ESTATE, "attention needs a preceding kvc_append_chunk (no evict/release after it)");
+  if (!((ctx->layers_written >> layer) & 1))
+    return fail(KVC_ESTATE, "layer %d's K/V of the last append are not written (kvc_append_kv_layer)",
+                layer);
   return KVC_OK;
 }
 

@@ -398,6 +398,8 @@ struct SeqArgs {
 cudaError_t launch_init(const Dev& d, double rope_base, cudaStream_t s);
 cudaError_t launch_append(const Dev& d, const AppendArgs& a, const uint8_t* types, const void* k,
                           const void* v, cudaStream_t s);
+cudaError_t launch_append_layers(const Dev& d, int total, int layer0, int n_layers, const void* k,
+                                 const void* v, cudaStream_t s);
 cudaError_t launch_evict(const Dev& d, const SeqArgs& a, int64_t* resident_out, cudaStream_t s);
 cudaError_t launch_release(const Dev& d, const SeqArgs& a, cudaStream_t s);
 cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_out, void* k_out,

@@ -336,16 +336,17 @@ __global__ void __launch_bounds__(META_THREADS) append_plan_kernel(Dev d, Append
 // the binary32 table), V copied, both into the page slots of part 1.
 // grid = (tokens, layers); K/V input layout [L][total][Hkv][D].
 template <typename T>
-__global__ void __launch_bounds__(256) append_kv_kernel(Dev d, int total, const T* k,
+__global__ void __launch_bounds__(256) append_kv_kernel(Dev d, int total, int layer0, const T* k,
                                                         const T* v) {
-  const int g = blockIdx.x, l = blockIdx.y;
+  // Input layer blockIdx.y of k/v is cache layer layer0 + blockIdx.y.
+  const int g = blockIdx.x, l = layer0 + blockIdx.y;
   if (g >= d.g->total_tokens) return;  // the plan kernel failed (device error recorded)
   const int D = d.head_dim, half = D / 2, H = d.kv_heads;
   const int gs = d.tok_slot[g];
   const int pos = d.tok_pos[g];
   const int page = gs / PS, slot = gs % PS;
-  const T* kin = k + ((size_t)l * total + g) * H * D;
-  const T* vin = v + ((size_t)l * total + g) * H * D;
+  const T* kin = k + ((size_t)blockIdx.y * total + g) * H * D;
+  const T* vin = v + ((size_t)blockIdx.y * total + g) * H * D;
   T* pool = reinterpret_cast<T*>(d.pool);
   const float2* cs = d.rope + (size_t)pos * half;
   for (int idx = threadIdx.x; idx < H * half; idx += blockDim.x) {
@@ -771,12 +772,19 @@ cudaError_t launch_init(const Dev& d, double rope_base, cudaStream_t s) {
 cudaError_t launch_append(const Dev& d, const AppendArgs& a, const uint8_t* types, const void* k,
                           const void* v, cudaStream_t s) {
   append_plan_kernel<<<1, META_THREADS, 0, s>>>(d, a, types);
-  dim3 grid(a.total, d.layers);
+  if (k == nullptr) return cudaGetLastError();  // plan only: layers follow one by one
+  return launch_append_layers(d, a.total, 0, d.layers, k, v, s);
+}
+
+cudaError_t launch_append_layers(const Dev& d, int total, int layer0, int n_layers, const void* k,
+                                 const void* v, cudaStream_t s) {
+  dim3 grid(total, n_layers);
   if (d.esz == 2)
     append_kv_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(
-        d, a.total, static_cast<const __nv_bfloat16*>(k), static_cast<const __nv_bfloat16*>(v));
+        d, total, layer0, static_cast<const __nv_bfloat16*>(k),
+        static_cast<const __nv_bfloat16*>(v));
   else
-    append_kv_kernel<float><<<grid, 256, 0, s>>>(d, a.total, static_cast<const float*>(k),
+    append_kv_kernel<float><<<grid, 256, 0, s>>>(d, total, layer0, static_cast<const float*>(k),
                                                  static_cast<const float*>(v));
   return cudaGetLastError();
 }

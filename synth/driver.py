@@ -174,18 +174,28 @@ class Driver:
 
     # -- API calls ---------------------------------------------------------------------------
     def run_call(self, c: Call, attention: bool = True, on_attention=None,
-                 on_append=None) -> int:
-        """Append + (optionally) every layer's attention. Returns kernels launched."""
+                 on_append=None, per_layer: bool = False) -> int:
+        """Append + (optionally) every layer's attention. Returns kernels launched.
+
+        per_layer: the model's order; the append carries no K/V and each layer's K/V
+        are written just before that layer's attention."""
         cache = self.cache
         _, s_p, _, c_p, t_ptr, k_ptr, v_ptr, q_ptrs, o_ptr = c.raw
-        cache.append_chunk_raw(len(c.sessions), s_p, c_p, t_ptr, k_ptr, v_ptr, self.stream)
+        stream = self.stream
+        cache.append_chunk_raw(len(c.sessions), s_p, c_p, t_ptr, None if per_layer else k_ptr,
+                               None if per_layer else v_ptr, stream)
         if on_append is not None:
             on_append(c)
-        launches = 2
-        if attention and c.q is not None and c.kind != "prefix":
-            fn = cache.attn_prefill_raw if c.kind == "prefill" else cache.attn_decode_raw
-            stream = self.stream
-            for layer in range(self.w.layers):
+        launches = 1 if per_layer else 2
+        do_attn = attention and c.q is not None and c.kind != "prefix"
+        fn = cache.attn_prefill_raw if c.kind == "prefill" else cache.attn_decode_raw
+        kv_stride = c.k.stride(0) * c.k.element_size()
+        for layer in range(self.w.layers):
+            if per_layer:
+                cache.append_kv_layer_raw(layer, k_ptr + layer * kv_stride,
+                                          v_ptr + layer * kv_stride, stream)
+                launches += 1
+            if do_attn:
                 fn(layer, q_ptrs[layer], o_ptr, stream)
                 launches += 1
                 if on_attention is not None:
@@ -193,10 +203,10 @@ class Driver:
         return launches
 
     def run_step(self, st: Step, attention: bool = True, on_attention=None,
-                 on_evict=None, on_append=None) -> int:
+                 on_evict=None, on_append=None, per_layer: bool = False) -> int:
         launches = 0
         for c in st.calls:
-            launches += self.run_call(c, attention, on_attention, on_append)
+            launches += self.run_call(c, attention, on_attention, on_append, per_layer)
         if st.evict_sessions is not None and len(st.evict_sessions):
             self.cache.evict(st.evict_sessions, self.resident_out)
             launches += 2

@@ -60,7 +60,7 @@ class Lockstep:
                               w.dtype, w.q_scale)
 
     def run_step(self, attn_pred=None, session_pred=None, check_state=True,
-                 state_sessions=None):
+                 state_sessions=None, per_layer=False):
         """One duplex step on both sides.
 
         attn_pred(step, call_kind, call_index, layer) -> bool selects attention calls to
@@ -106,5 +106,5 @@ class Lockstep:
                               f"step {step.index} session {s}")
 
         self.drv.run_step(st, attention=True, on_attention=on_attention, on_evict=on_evict,
-                          on_append=on_append)
+                          on_append=on_append, per_layer=per_layer)
         return st

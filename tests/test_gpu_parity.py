@@ -157,6 +157,35 @@ def test_transcript_export():
         assert torch.equal(k2[:, :3], k[:, :3])
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_per_layer_append(dtype):
+    """The model's order: appends without K/V, each layer's K/V written just before that
+    layer's attention; state and every output as with whole-chunk appends."""
+    w = (S.SINGLE_BF16.with_(layers=3, n_sessions=3, budget=80, window=2, seed=13,
+                             turn_period=10, turn_jitter=1) if dtype == "bf16"
+         else S.TINY_F32.with_(units=30))
+    ls, _ = _lockstep(w, n_units=30)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda *a: True, per_layer=True)
+    assert ls.n_compared > 0
+
+
+def test_attention_needs_the_layer_written():
+    from paper_2609_31224_gb300._lib import KvcError
+    w = S.SINGLE_BF16.with_(layers=2, n_sessions=1, units=3)
+    drv = Driver(w, S.workload_scripts(w))
+    st = drv.prepare_step()
+    c = [c for c in st.calls if c.kind == "prefill"][0]
+    drv.cache.append_chunk(c.sessions, c.cu, c.types, None, None)
+    with pytest.raises(KvcError, match="ESTATE"):
+        drv.cache.attn_prefill_chunk(0, c.q[0], c.out)
+    drv.cache.append_kv_layer(0, c.k[0], c.v[0])
+    drv.cache.attn_prefill_chunk(0, c.q[0], c.out)
+    with pytest.raises(KvcError, match="ESTATE"):
+        drv.cache.attn_prefill_chunk(1, c.q[1], c.out)
+    torch.cuda.synchronize()
+
+
 def test_sharp_attention_bf16():
     """Larger query scale makes the softmax peaked, so a wrong key order shows.
 
