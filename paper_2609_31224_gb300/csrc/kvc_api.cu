@@ -35,7 +35,7 @@ int fail(int code, const char* fmt, ...) {
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Sizes {
-  int max_moves, max_alloc, max_dec_items, max_pf_items;
+  int max_moves, max_alloc, dec_slots, max_pf_items;
 };
 
 Sizes derive_sizes(const kvc_config& c) {
@@ -44,7 +44,7 @@ Sizes derive_sizes(const kvc_config& c) {
   s.max_moves = (int)std::min<int64_t>(mv, 1 << 26);
   s.max_alloc = s.max_moves / PS + c.max_tokens_per_call / PS + 2 * c.max_seq_per_call + 1;
   // Decode partial slots: two per CTA of the stream-K split (grid <= 2048 CTAs).
-  s.max_dec_items = 4096;
+  s.dec_slots = 4096;
   // Prefill partial slots: the binary32 kernel's chunk list, and two per CTA of the
   // bfloat16 kernel's stream-K split.
   s.max_pf_items = (int)std::min<int64_t>(2048, std::max<int64_t>(512, (int64_t)c.max_seq_per_call * c.kv_heads * 4));
@@ -75,14 +75,13 @@ size_t layout_meta(const kvc_config& c, uint8_t* base, Dev* d) {
   uint8_t* glob = take(sizeof(DevGlobals));
   uint8_t* rope = take((size_t)c.max_positions * (c.head_dim / 2) * sizeof(float2));
   uint8_t* seq = take((size_t)c.max_seq_per_call * sizeof(SeqInfo));
-  uint8_t* di = take((size_t)z.max_dec_items * sizeof(Item));
   uint8_t* pi = take((size_t)z.max_pf_items * sizeof(Item));
   uint8_t* ts = take((size_t)c.max_tokens_per_call * 4);
   uint8_t* tp = take((size_t)c.max_tokens_per_call * 4);
   uint8_t* mv = take((size_t)z.max_moves * sizeof(int2));
   uint8_t* al = take((size_t)z.max_alloc * 4);
-  uint8_t* dpo = take((size_t)z.max_dec_items * G * c.head_dim * 4);
-  uint8_t* dpm = take((size_t)z.max_dec_items * G * sizeof(float2));
+  uint8_t* dpo = take((size_t)z.dec_slots * G * c.head_dim * 4);
+  uint8_t* dpm = take((size_t)z.dec_slots * G * sizeof(float2));
   uint8_t* ppo = take((size_t)z.max_pf_items * PF_MAX_TOKENS * G * 128 * 4);
   uint8_t* ppm = take((size_t)z.max_pf_items * PF_MAX_TOKENS * G * sizeof(float2));
   uint8_t* dc = take((size_t)c.max_seq_per_call * c.kv_heads * 4);
@@ -99,7 +98,6 @@ size_t layout_meta(const kvc_config& c, uint8_t* base, Dev* d) {
     d->g = reinterpret_cast<DevGlobals*>(glob);
     d->rope = reinterpret_cast<float2*>(rope);
     d->seq = reinterpret_cast<SeqInfo*>(seq);
-    d->dec_items = reinterpret_cast<Item*>(di);
     d->pf_items = reinterpret_cast<Item*>(pi);
     d->tok_slot = reinterpret_cast<int32_t*>(ts);
     d->tok_pos = reinterpret_cast<int32_t*>(tp);
@@ -113,7 +111,7 @@ size_t layout_meta(const kvc_config& c, uint8_t* base, Dev* d) {
     d->pf_count = reinterpret_cast<int32_t*>(pc);
     d->max_moves = z.max_moves;
     d->max_alloc = z.max_alloc;
-    d->max_dec_items = z.max_dec_items;
+    d->dec_slots = z.dec_slots;
     d->max_pf_items = z.max_pf_items;
     d->bitmap_words = words;
   }
@@ -332,9 +330,7 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, const i
   AppendArgs a;
   a.n_seq = n_seq;
   a.total = total;
-  a.dec_target = 0;  // decode uses the stream-K split
   a.pf_target = ctx->pf_target;
-  a.dec_min_blocks = 0;
   a.pf_min_blocks = 4;
   for (int i = 0; i < n_seq; ++i) a.sessions[i] = h_sessions[i];
   for (int i = 0; i <= n_seq; ++i) a.cu[i] = h_cu_tokens[i];

@@ -669,7 +669,7 @@ int stream_k_grid(const Dev& d) {
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   // Every CTA of the stream-K split may write two partial slots.
-  return min(d.max_dec_items / 2, max(1, per_sm) * sms);
+  return min(d.dec_slots / 2, max(1, per_sm) * sms);
 }
 
 // Resident CTAs of the pair-split kernel (one wave).

@@ -45,7 +45,7 @@ struct SeqInfo {
   int32_t live_head;
   int32_t n_live;
   int32_t n_blocks;     // n_hist_pages + n_live_pages
-  int32_t dec_chunks;   // unused (attention splits the call's units, see UnitSplit)
+  int32_t pad0;
   int32_t unit_base;    // first (session, kv head, page) unit of this session
   int32_t pf_chunks;
   int32_t pf_base;
@@ -85,7 +85,8 @@ struct Dev {
   int64_t n_pages;
   int32_t bitmap_words;
   int32_t max_moves;
-  int32_t max_dec_items, max_pf_items;   // items including the kv-head factor
+  int32_t dec_slots;           // decode partial slots (two per CTA of a split)
+  int32_t max_pf_items;        // prefill chunk items (binary32) / partial slots (bfloat16)
   // memory
   uint8_t* pool;
   SessState* sess;
@@ -98,15 +99,14 @@ struct Dev {
   DevGlobals* g;
   float2* rope;                // [max_positions][D/2] (cos, sin)
   SeqInfo* seq;                // [max_seq]
-  Item* dec_items;             // [max_dec_items]
   Item* pf_items;              // [max_pf_items]
   int32_t* tok_slot;           // [max_tokens] page * PS + slot
   int32_t* tok_pos;            // [max_tokens]
   int2* moves;                 // [max_moves] (src page*PS+slot, dst page*PS+slot)
   int32_t* alloc_list;         // [max_alloc] pages handed out by the last allocation
   int32_t max_alloc;
-  float* dec_part_o;           // [max_dec_items][G][D]
-  float2* dec_part_ml;         // [max_dec_items][G] (m, l) in log2 units
+  float* dec_part_o;           // [dec_slots][G][D]
+  float2* dec_part_ml;         // [dec_slots][G] (m, l) in log2 units
   float* pf_part_o;            // [max_pf_items][PF_ROWS][D]
   float2* pf_part_ml;          // [max_pf_items][PF_ROWS]
   int32_t* dec_count;          // [max_seq * kv_heads] arrival counters
@@ -384,8 +384,8 @@ __device__ inline float exp2_safe(float x, float m) {
 struct AppendArgs {
   int32_t n_seq;
   int32_t total;
-  int32_t dec_target, pf_target;   // desired split-K item counts
-  int32_t dec_min_blocks, pf_min_blocks;
+  int32_t pf_target;       // desired item count of the binary32 prefill's chunk list
+  int32_t pf_min_blocks;
   int32_t sessions[MAX_SEQ];
   int32_t cu[MAX_SEQ + 1];
 };

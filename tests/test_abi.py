@@ -88,7 +88,22 @@ def test_null_context_is_rejected(lib):
     assert lib.kvc_attn_decode(None, 0, None, None, None) == -1
     out = ctypes.c_int64()
     assert lib.kvc_resident_size(None, 0, ctypes.byref(out)) == -1
+    assert lib.kvc_append_kv_layer(None, 0, None, None, None) == -1
+    assert lib.kvc_export_transcript(None, 0, 0, None, None, None, None, None) == -1
+    assert lib.kvc_last_error()
     lib.kvc_destroy(None)
+
+
+def test_policy_fields_are_validated(lib):
+    pool, meta = ctypes.c_size_t(), ctypes.c_size_t()
+    for bad in ({"policy": 3}, {"policy": -1}, {"policy": 2, "sink": -1},
+                {"policy": 2, "recent": -5}):
+        assert lib.kvc_query_sizes(ctypes.byref(_cfg(**bad)), ctypes.byref(pool),
+                                   ctypes.byref(meta)) == -1
+        assert b"policy" in lib.kvc_last_error() or b"sink" in lib.kvc_last_error()
+    for good in ({"policy": 1}, {"policy": 2, "sink": 4, "recent": 2000}):
+        assert lib.kvc_query_sizes(ctypes.byref(_cfg(**good)), ctypes.byref(pool),
+                                   ctypes.byref(meta)) == 0
 
 
 def test_synth_generator_builds():
