@@ -219,24 +219,24 @@ def run_ours(args, rank: int, world: int, local_rank: int):
                 dec_ev[i][1].record(stream)
                 launches += 2 + w.layers
             elif c is first_dec:
-                # The model's order: each layer's K/V written just before its attention;
-                # each decode launch is timed on its own.
+                # The model's order: each layer's K/V written by its own decode launch
+                # (fused); each launch is timed on its own.
                 _, s_p, _, c_p, t_ptr, k_ptr, v_ptr, q_ptrs, o_ptr = c.raw
                 drv.cache.append_chunk_raw(len(c.sessions), s_p, c_p, t_ptr, None, None,
                                            drv.stream)
                 kv_stride = c.k.stride(0) * c.k.element_size()
                 evs = []
                 for layer in range(w.layers):
-                    drv.cache.append_kv_layer_raw(layer, k_ptr + layer * kv_stride,
-                                                  v_ptr + layer * kv_stride, drv.stream)
                     e0 = torch.cuda.Event(enable_timing=True)
                     e1 = torch.cuda.Event(enable_timing=True)
                     e0.record(stream)
-                    drv.cache.attn_decode_raw(layer, q_ptrs[layer], o_ptr, drv.stream)
+                    drv.cache.attn_decode_kv_raw(layer, k_ptr + layer * kv_stride,
+                                                 v_ptr + layer * kv_stride, q_ptrs[layer], o_ptr,
+                                                 drv.stream)
                     e1.record(stream)
                     evs.append((e0, e1))
                 dec_ev[i] = evs
-                launches += 1 + 2 * w.layers
+                launches += 1 + w.layers
             else:
                 launches += drv.run_call(c, per_layer=per_layer)
         drv.cache.evict(st.evict_sessions, drv.resident_out)

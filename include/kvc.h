@@ -164,6 +164,16 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions,
  *   d_k, d_v   device [total][Hkv][D], total and order as in the last append */
 int kvc_append_kv_layer(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v, void* stream);
 
+/* Decode attention of one layer fused with that layer's K/V write (the
+ * per-layer order, after kvc_append_chunk without K/V): the new tokens' K
+ * (rotated at their positions) and V of the layer are written into their slots
+ * and attended in the same launch.  Same results and stored bytes as
+ * kvc_append_kv_layer followed by kvc_attn_decode.
+ *   d_k, d_v   device [n_seq][Hkv][D], the layer's rows of the appended tokens
+ *   other arguments as for kvc_attn_decode */
+int kvc_attn_decode_kv(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v,
+                       const void* d_q, void* d_out, void* stream);
+
 /* Online eviction (Sec. 3.3) for each listed session, run by the caller after
  * a unit: while resident > B, evict the ACOUSTIC and ASR_DELIM positions of
  * the oldest unit u with 0 <= u <= unit_cur - W that still has some; stop

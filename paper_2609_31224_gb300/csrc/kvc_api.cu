@@ -408,7 +408,8 @@ int kvc_release(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, void* stream
   return KVC_OK;
 }
 
-static int check_attn(kvc_ctx* ctx, int layer, const void* d_q, void* d_out) {
+static int check_attn(kvc_ctx* ctx, int layer, const void* d_q, void* d_out,
+                      bool writes_layer = false) {
   if (!ctx) return fail(KVC_EINVAL, "ctx is NULL");
   if (layer < 0 || layer >= ctx->cfg.layers)
     return fail(KVC_EINVAL, "layer %d outside 0..%d", layer, ctx->cfg.layers - 1);
@@ -416,7 +417,7 @@ static int check_attn(kvc_ctx* ctx, int layer, const void* d_q, void* d_out) {
   if (!aligned16(d_q) || !aligned16(d_out)) return fail(KVC_EINVAL, "d_q / d_out must be 16-byte aligned");
   if (!ctx->attn_valid)
     return fail(KVC_ESTATE, "attention needs a preceding kvc_append_chunk (no evict/release after it)");
-  if (!((ctx->layers_written >> layer) & 1))
+  if (!writes_layer && !((ctx->layers_written >> layer) & 1))
     return fail(KVC_ESTATE, "layer %d's K/V of the last append are not written (kvc_append_kv_layer)",
                 layer);
   return KVC_OK;
@@ -432,6 +433,25 @@ int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void*
   // new token's K/V, so it does not start early; later ones may.
   KVC_CUDA(launch_attn_decode(ctx->d, layer, d_q, d_out, ctx->last_n_seq,
                               ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream)));
+  ++ctx->attn_since_append;
+  return KVC_OK;
+}
+
+int kvc_attn_decode_kv(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v,
+                      const void* d_q, void* d_out, void* stream) {
+  g_err.clear();
+  int rc = check_attn(ctx, layer, d_q, d_out, true);
+  if (rc) return rc;
+  if (!d_k || !d_v) return fail(KVC_EINVAL, "d_k / d_v must be non-NULL");
+  if (!aligned16(d_k) || !aligned16(d_v)) return fail(KVC_EINVAL, "d_k / d_v must be 16-byte aligned");
+  if (!ctx->last_single)
+    return fail(KVC_ESTATE, "decode needs exactly one appended token per session");
+  // Launches after the append may start early: the new rows go into the tiles
+  // after their loads, and the previous launch writes another layer's rows only.
+  KVC_CUDA(launch_attn_decode(ctx->d, layer, d_q, d_out, ctx->last_n_seq,
+                              ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream), d_k,
+                              d_v));
+  ctx->layers_written |= 1ull << layer;
   ++ctx->attn_since_append;
   return KVC_OK;
 }

@@ -201,13 +201,52 @@ __device__ void load_q(const Dev& d, const SeqInfo& si, int head, const typename
   }
 }
 
+// Fused layer write (per-layer order): the session's new token K (rotated at its
+// position, the append kernel's binary32 arithmetic) and V of this layer and head,
+// read from the caller's [total][Hkv][D] rows, go into the pool slot and into the
+// K/V tile just loaded from it (whose copy of that row may be stale).  Called by
+// the warp that streams the pair's last block, which holds the token.
+template <class C>
+__device__ void patch_new_row(const Dev& d, int layer, const SeqInfo& si, int head,
+                              const typename C::T* nk, const typename C::T* nv, uint8_t* kt,
+                              int lane) {
+  using T = typename C::T;
+  constexpr int D = C::D, HALF = D / 2;
+  const int gs = d.tok_slot[si.q_row0];
+  const int page = gs / PS, slot = gs % PS;
+  const T* kin = nk + ((size_t)si.q_row0 * d.kv_heads + head) * D;
+  const T* vin = nv + ((size_t)si.q_row0 * d.kv_heads + head) * D;
+  const float2* cs = d.rope + (size_t)si.pos_first * HALF;
+  T* kp = reinterpret_cast<T*>(d.pool) + pool_offset_elems(d, page, layer, 0, head, slot);
+  T* vp = reinterpret_cast<T*>(d.pool) + pool_offset_elems(d, page, layer, 1, head, slot);
+  T* kr = reinterpret_cast<T*>(kt + slot * C::ROW_BYTES);
+  T* vr = reinterpret_cast<T*>(kt + C::TILE + slot * C::ROW_BYTES);
+  for (int j = lane; j < HALF; j += 32) {
+    const float x1 = to_float<T>(kin[j]), x2 = to_float<T>(kin[j + HALF]);
+    const float2 c = cs[j];
+    const T y1 = from_float<T>(fmaf(x1, c.x, -x2 * c.y));
+    const T y2 = from_float<T>(fmaf(x2, c.x, x1 * c.y));
+    kr[j] = y1;
+    kr[j + HALF] = y2;
+    kp[j] = y1;
+    kp[j + HALF] = y2;
+  }
+  for (int j = lane; j < D; j += 32) {
+    const T x = vin[j];
+    vr[j] = x;
+    vp[j] = x;
+  }
+  __syncwarp();
+}
+
 // Stream this warp's blocks of the segment: scores, online softmax, P V.  The first
 // STAGES blocks must have been issued (Segment::prefetch).  Returns the first block
 // whose wait gave up, or -1.
-template <class C>
+template <class C, bool FUSED>
 __device__ int stream_pages(const Dev& d, int layer, Segment<C>& sg, const Smem<C>& sm,
                             uint32_t loads, const float (&qr)[G][2 * C::VEC], float& m_run,
-                            float& l_run, float2 (&acc)[G][C::PVD / 2], int warp, int lane) {
+                            float& l_run, float2 (&acc)[G][C::PVD / 2], int warp, int lane,
+                            const typename C::T* new_k, const typename C::T* new_v) {
   using T = typename C::T;
   const int kq = lane >> 3, c = lane & 7;
   const bool up4 = lane & 4, up2 = lane & 2;
@@ -218,7 +257,13 @@ __device__ int stream_pages(const Dev& d, int layer, Segment<C>& sg, const Smem<
     if (!__all_sync(FULL, mbar_wait(d, &sm.wbars[st], (n / C::STAGES) & 1))) return k;
     const uint8_t* kt = sm.tiles + st * 2 * C::TILE;
     const uint8_t* vt = kt + C::TILE;
-    const BlockRange br = block_range(sg.si, sg.blk_begin + warp + k * C::WARPS);
+    const int blk = sg.blk_begin + warp + k * C::WARPS;
+    if constexpr (FUSED) {
+      if (blk == sg.si.n_blocks - 1)
+        patch_new_row<C>(d, layer, sg.si, sg.head, new_k, new_v, sm.tiles + st * 2 * C::TILE,
+                         lane);
+    }
+    const BlockRange br = block_range(sg.si, blk);
     const bool interior = br.lo == 0 && br.hi == PS;
 
     // Scores: the 8 lanes 8j..8j+7 take key 4i + j, lane c its chunks c and c + 8.
@@ -490,10 +535,10 @@ __device__ void merge_parts(const Dev& d, const Smem<C>& sm, int nch, PartFn par
 // ---------------------------------------------------------------------------
 // Stream-K kernel.
 // ---------------------------------------------------------------------------
-template <typename T, int D>
+template <typename T, int D, bool FUSED>
 __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
     Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale,
-    int min_units) {
+    int min_units, const T* new_k, const T* new_v) {
   using C = SkCfg<T, D>;
   static_assert(C::WARPS == G, "the split-K merge maps one warp to one query row");
   extern __shared__ __align__(128) uint8_t smem[];
@@ -539,8 +584,8 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
     for (int g = 0; g < G; ++g)
 #pragma unroll
       for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
-    const int failed_at = stream_pages<C>(d, layer, sg, sm, loads, qr, m_run, l_run, acc, warp,
-                                          lane);
+    const int failed_at = stream_pages<C, FUSED>(d, layer, sg, sm, loads, qr, m_run, l_run, acc,
+                                                 warp, lane, new_k, new_v);
     if (failed_at >= 0 && lane == 0) s_abort = 1;
     __syncthreads();
     if (s_abort) {
@@ -596,9 +641,10 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
 // waits on the previous kernel; the k partial states of a pair are merged by
 // the last of its CTAs to finish.
 // ---------------------------------------------------------------------------
-template <typename T, int D>
+template <typename T, int D, bool FUSED>
 __global__ void __launch_bounds__(SpCfg<T, D>::THREADS, 1) attn_decode_split_kernel(
-    Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale, int k) {
+    Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale, int k,
+    const T* new_k, const T* new_v) {
   using C = SpCfg<T, D>;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -626,7 +672,8 @@ __global__ void __launch_bounds__(SpCfg<T, D>::THREADS, 1) attn_decode_split_ker
   for (int g = 0; g < G; ++g)
 #pragma unroll
     for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
-  const int failed_at = stream_pages<C>(d, layer, sg, sm, 0, qr, m_run, l_run, acc, warp, lane);
+  const int failed_at = stream_pages<C, FUSED>(d, layer, sg, sm, 0, qr, m_run, l_run, acc, warp,
+                                               lane, new_k, new_v);
   if (failed_at >= 0) {
     // A wait gave up (error recorded): drain this warp's copies, contribute nothing.
     for (int j = failed_at; j < min(sg.n_my, failed_at + C::STAGES); ++j)
@@ -660,9 +707,11 @@ __global__ void __launch_bounds__(SpCfg<T, D>::THREADS, 1) attn_decode_split_ker
 // Resident CTAs of the stream-K kernel (its grid), capped by the partial slots.
 template <typename T, int D>
 int stream_k_grid(const Dev& d) {
-  const void* fn = reinterpret_cast<const void*>(&attn_decode_kernel<T, D>);
+  const void* fn = reinterpret_cast<const void*>(&attn_decode_kernel<T, D, false>);
   const int smem = SkCfg<T, D>::SMEM;
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_decode_kernel<T, D, true>),
+                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   int per_sm = 0;
   cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SkCfg<T, D>::THREADS, smem);
   int dev = 0, sms = 0;
@@ -675,9 +724,11 @@ int stream_k_grid(const Dev& d) {
 // Resident CTAs of the pair-split kernel (one wave).
 template <typename T, int D>
 int split_slots() {
-  const void* fn = reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D>);
+  const void* fn = reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D, false>);
   const int smem = SpCfg<T, D>::SMEM;
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D, true>),
+                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   int per_sm = 0;
   cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SpCfg<T, D>::THREADS, smem);
   int dev = 0, sms = 0;
@@ -694,28 +745,34 @@ constexpr int SPLIT_MIN_K = 2;
 
 template <typename T, int D>
 cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int n_seq, bool pdl,
-                          cudaStream_t s) {
+                          cudaStream_t s, const void* new_k, const void* new_v) {
   static thread_local const int grid = stream_k_grid<T, D>(d);
   static thread_local const int slots = split_slots<T, D>();
   const float scale = LOG2E / sqrtf((float)D);
   const int n_pairs = n_seq * d.kv_heads;
   const T* qt = static_cast<const T*>(q);
   T* ot = static_cast<T*>(out);
+  const T* nk = static_cast<const T*>(new_k);
+  const T* nv = static_cast<const T*>(new_v);
   const int k = n_pairs * SPLIT_MIN_K <= slots ? min(MAX_PARTS, slots / n_pairs) : 0;
+  const bool fused = nk != nullptr;
   if (k > 0)
-    return launch_ex(&attn_decode_split_kernel<T, D>, dim3(n_pairs * k),
-                     dim3(SpCfg<T, D>::THREADS), SpCfg<T, D>::SMEM, s, pdl, d, layer, qt, ot,
-                     scale, k);
-  return launch_ex(&attn_decode_kernel<T, D>, dim3(grid), dim3(SkCfg<T, D>::THREADS),
-                   SkCfg<T, D>::SMEM, s, pdl, d, layer, qt, ot, scale, DEC_MIN_UNITS);
+    return launch_ex(fused ? &attn_decode_split_kernel<T, D, true>
+                           : &attn_decode_split_kernel<T, D, false>,
+                     dim3(n_pairs * k), dim3(SpCfg<T, D>::THREADS), SpCfg<T, D>::SMEM, s, pdl, d,
+                     layer, qt, ot, scale, k, nk, nv);
+  return launch_ex(fused ? &attn_decode_kernel<T, D, true> : &attn_decode_kernel<T, D, false>,
+                   dim3(grid), dim3(SkCfg<T, D>::THREADS), SkCfg<T, D>::SMEM, s, pdl, d, layer,
+                   qt, ot, scale, DEC_MIN_UNITS, nk, nv);
 }
 
 }  // namespace
 
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               bool pdl, cudaStream_t s) {
-  if (d.esz == 2) return launch_decode<__nv_bfloat16, 128>(d, layer, q, out, n_seq, pdl, s);
-  return launch_decode<float, 64>(d, layer, q, out, n_seq, pdl, s);
+                               bool pdl, cudaStream_t s, const void* new_k, const void* new_v) {
+  if (d.esz == 2)
+    return launch_decode<__nv_bfloat16, 128>(d, layer, q, out, n_seq, pdl, s, new_k, new_v);
+  return launch_decode<float, 64>(d, layer, q, out, n_seq, pdl, s, new_k, new_v);
 }
 
 }  // namespace kvc

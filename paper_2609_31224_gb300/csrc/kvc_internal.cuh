@@ -404,8 +404,10 @@ cudaError_t launch_evict(const Dev& d, const SeqArgs& a, int64_t* resident_out, 
 cudaError_t launch_release(const Dev& d, const SeqArgs& a, cudaStream_t s);
 cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_out, void* k_out,
                               void* v_out, int32_t* count, cudaStream_t s);
+// new_k / new_v (optional): the fused per-layer write of the new tokens' K/V.
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               bool pdl, cudaStream_t s);
+                               bool pdl, cudaStream_t s, const void* new_k = nullptr,
+                               const void* new_v = nullptr);
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                 int max_t, bool pdl, cudaStream_t s);
 cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,

@@ -191,9 +191,16 @@ class Driver:
         fn = cache.attn_prefill_raw if c.kind == "prefill" else cache.attn_decode_raw
         kv_stride = c.k.stride(0) * c.k.element_size()
         for layer in range(self.w.layers):
+            kl, vl = k_ptr + layer * kv_stride, v_ptr + layer * kv_stride
+            if per_layer and do_attn and c.kind == "decode":
+                # The layer's K/V write fused into its decode launch.
+                cache.attn_decode_kv_raw(layer, kl, vl, q_ptrs[layer], o_ptr, stream)
+                launches += 1
+                if on_attention is not None:
+                    on_attention(c, layer)
+                continue
             if per_layer:
-                cache.append_kv_layer_raw(layer, k_ptr + layer * kv_stride,
-                                          v_ptr + layer * kv_stride, stream)
+                cache.append_kv_layer_raw(layer, kl, vl, stream)
                 launches += 1
             if do_attn:
                 fn(layer, q_ptrs[layer], o_ptr, stream)

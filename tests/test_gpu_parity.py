@@ -170,6 +170,28 @@ def test_per_layer_append(dtype):
     assert ls.n_compared > 0
 
 
+def test_fused_layer_write_stores_the_same_bytes():
+    """Whole-chunk appends and the per-layer order (separate writes for prefill chunks,
+    writes fused into the decode launches) leave bit-identical K/V in every layer."""
+    w = S.SINGLE_BF16.with_(layers=3, n_sessions=2, budget=60, window=1, seed=3,
+                            turn_period=8, turn_jitter=1)
+    scripts = S.workload_scripts(w)
+    for sc in scripts:
+        sc.n_transcript = sc.n_transcript[:25]
+        sc.n_text = sc.n_text[:25]
+    a, b = Driver(w, scripts), Driver(w, scripts)
+    for _ in range(len(a.sched)):
+        a.run_step(a.prepare_step())
+        b.run_step(b.prepare_step(), per_layer=True)
+    torch.cuda.synchronize()
+    for s in range(2):
+        assert a.cache.export_state(s)["pos"] == b.cache.export_state(s)["pos"]
+        for layer in range(w.layers):
+            ka, va = a.cache.export_kv(s, layer)
+            kb, vb = b.cache.export_kv(s, layer)
+            assert np.array_equal(ka, kb) and np.array_equal(va, vb)
+
+
 def test_attention_needs_the_layer_written():
     from paper_2609_31224_gb300._lib import KvcError
     w = S.SINGLE_BF16.with_(layers=2, n_sessions=1, units=3)
