@@ -641,11 +641,10 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
 // waits on the previous kernel; the k partial states of a pair are merged by
 // the last of its CTAs to finish.
 // ---------------------------------------------------------------------------
-template <typename T, int D, bool FUSED>
-__global__ void __launch_bounds__(SpCfg<T, D>::THREADS, 1) attn_decode_split_kernel(
+template <typename T, int D, bool FUSED, class C>
+__global__ void __launch_bounds__(C::THREADS) attn_decode_split_kernel(
     Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale, int k,
     const T* new_k, const T* new_v) {
-  using C = SpCfg<T, D>;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const Smem<C> sm(smem, warp);
@@ -721,16 +720,16 @@ int stream_k_grid(const Dev& d) {
   return min(d.dec_slots / 2, max(1, per_sm) * sms);
 }
 
-// Resident CTAs of the pair-split kernel (one wave).
-template <typename T, int D>
+// Resident CTAs of the pair-split kernel with CTA shape C (one wave).
+template <typename T, int D, class C>
 int split_slots() {
-  const void* fn = reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D, false>);
-  const int smem = SpCfg<T, D>::SMEM;
+  const void* fn = reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D, false, C>);
+  const int smem = C::SMEM;
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D, true>),
+  cudaFuncSetAttribute(reinterpret_cast<const void*>(&attn_decode_split_kernel<T, D, true, C>),
                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   int per_sm = 0;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SpCfg<T, D>::THREADS, smem);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, C::THREADS, smem);
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -740,14 +739,16 @@ int split_slots() {
 // Minimum (session, kv head, page) units per CTA of the stream-K split.
 constexpr int DEC_MIN_UNITS = 12;
 // The pair-split kernel takes calls whose pairs each get at least this many CTAs
-// in one wave.
-constexpr int SPLIT_MIN_K = 2;
+// in one wave: with 16-warp CTAs (one per SM) first, else with stream-K's 4-warp
+// CTAs (three per SM).
+constexpr int SPLIT_MIN_K = 2, SPLIT4_MIN_K = 3;
 
 template <typename T, int D>
 cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int n_seq, bool pdl,
                           cudaStream_t s, const void* new_k, const void* new_v) {
   static thread_local const int grid = stream_k_grid<T, D>(d);
-  static thread_local const int slots = split_slots<T, D>();
+  static thread_local const int slots = split_slots<T, D, SpCfg<T, D>>();
+  static thread_local const int slots4 = split_slots<T, D, SkCfg<T, D>>();
   const float scale = LOG2E / sqrtf((float)D);
   const int n_pairs = n_seq * d.kv_heads;
   const T* qt = static_cast<const T*>(q);
@@ -756,11 +757,21 @@ cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int
   const T* nv = static_cast<const T*>(new_v);
   const int k = n_pairs * SPLIT_MIN_K <= slots ? min(MAX_PARTS, slots / n_pairs) : 0;
   const bool fused = nk != nullptr;
-  if (k > 0)
-    return launch_ex(fused ? &attn_decode_split_kernel<T, D, true>
-                           : &attn_decode_split_kernel<T, D, false>,
-                     dim3(n_pairs * k), dim3(SpCfg<T, D>::THREADS), SpCfg<T, D>::SMEM, s, pdl, d,
-                     layer, qt, ot, scale, k, nk, nv);
+  if (k > 0) {
+    using C = SpCfg<T, D>;
+    return launch_ex(fused ? &attn_decode_split_kernel<T, D, true, C>
+                           : &attn_decode_split_kernel<T, D, false, C>,
+                     dim3(n_pairs * k), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, qt, ot,
+                     scale, k, nk, nv);
+  }
+  const int k4 = n_pairs * SPLIT4_MIN_K <= slots4 ? min(MAX_PARTS, slots4 / n_pairs) : 0;
+  if (k4 > 0) {
+    using C = SkCfg<T, D>;
+    return launch_ex(fused ? &attn_decode_split_kernel<T, D, true, C>
+                           : &attn_decode_split_kernel<T, D, false, C>,
+                     dim3(n_pairs * k4), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, qt, ot,
+                     scale, k4, nk, nv);
+  }
   return launch_ex(fused ? &attn_decode_kernel<T, D, true> : &attn_decode_kernel<T, D, false>,
                    dim3(grid), dim3(SkCfg<T, D>::THREADS), SkCfg<T, D>::SMEM, s, pdl, d, layer,
                    qt, ot, scale, DEC_MIN_UNITS, nk, nv);
