@@ -59,6 +59,21 @@ def decode_traffic(alg_bytes_per_launch):
     return DECODE_TRAFFIC_RATIO * alg_bytes_per_launch
 
 
+def decode_kernel_label(w) -> str:
+    """Kernel that the library's dispatch gives a full-batch decode call of `w` (sessions
+    at full budget): the 16-warp pair split while every (session, KV head) pair gets two
+    one-CTA-per-SM slices, the 4-warp pair split while it gets three of the three CTAs
+    per SM, else stream-K."""
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    pairs = w.n_sessions * w.kv_heads
+    if 2 * pairs <= sms:
+        return "attn_decode_split_kernel (16 warps)"
+    if pairs <= sms:
+        return "attn_decode_split_kernel (4 warps)"
+    return "attn_decode_kernel"
+
+
 def load_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -305,7 +320,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         "path_hbm_gbs": (tot_bytes / 1e9) / (elapsed_ms / 1e3),
         "path_frac_of_peak": (tot_bytes / 1e9) / (elapsed_ms / 1e3) / peak,
         "roofline": {
-            "kernel": "attn_decode_kernel",
+            "kernel": decode_kernel_label(w),
             "bound": "hbm",
             "achieved": dec_gbs,
             "peak": peak,
@@ -313,8 +328,8 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "unit": "GB/s",
             "frac": (dec_gbs / peak) if dec_gbs else None,
             "traffic": decode_traffic((sum(dec_bytes) / len(dec_bytes)) if dec_bytes else None),
-            "traffic_note": "ncu DRAM bytes per algorithmic byte on the 16-session reduced "
-                            "case, scaled to this launch",
+            "traffic_note": "ncu DRAM bytes per algorithmic byte of the stream-K kernel on "
+                            "the 24-session reduced case, scaled to this launch",
             "algorithmic_bytes_per_launch": (sum(dec_bytes) / len(dec_bytes)) if dec_bytes else None,
             "avg_launch_us": (1e3 * sum(dec_times) / len(dec_times)) if dec_times else None,
         },
@@ -351,23 +366,32 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
-    # Inputs move on a copy stream, step by step in order; each step's compute waits
-    # only for its own inputs, so transfers of later steps overlap earlier compute.
+    # Inputs move on a copy stream, one step ahead of the compute: step i+1's copies are
+    # enqueued just before step i's launches, and each step's compute waits only for its
+    # own inputs, so transfers overlap the previous step's compute.
     copy_stream = torch.cuda.Stream()
-    ready = [torch.cuda.Event() for _ in steps]
+    copy_start = [torch.cuda.Event(enable_timing=True) for _ in steps]
+    ready = [torch.cuda.Event(enable_timing=True) for _ in steps]
     t0 = time.perf_counter()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     copy_stream.wait_stream(stream)
     h2d_total, d2h_total = 0, 0
-    with torch.cuda.stream(copy_stream):
-        for si in range(len(steps)):
+
+    def enqueue_copies(si):
+        nonlocal h2d_total
+        with torch.cuda.stream(copy_stream):
+            copy_start[si].record(copy_stream)
             for ci in range(len(steps[si].calls)):
                 for n, t in host[si][ci].items():
                     dev[si][ci][n].copy_(t, non_blocking=True)
                     h2d_total += t.numel() * t.element_size()
             ready[si].record(copy_stream)
+
+    enqueue_copies(0)
     for si, st in enumerate(steps):
+        if si + 1 < len(steps):
+            enqueue_copies(si + 1)
         stream.wait_event(ready[si])
         for ci, c in enumerate(st.calls):
             drv.run_call(c, per_layer=per_layer)
@@ -379,9 +403,11 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
         res_host[:n].copy_(drv.resident_out[:n], non_blocking=True)
         d2h_total += n * 8
     e1.record(stream)
+    submit = time.perf_counter() - t0
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
     wall = time.perf_counter() - t0
+    copy_ms = [a.elapsed_time(b) for a, b in zip(copy_start, ready)]
     if world > 1:
         tt = torch.tensor([ms], dtype=torch.float64, device="cuda")
         torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
@@ -389,7 +415,10 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
     audio_s = sum(len(st.pairs) for st in steps)
     return {"value": world * audio_s / (ms / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d_total / n_steps, "d2h_bytes_per_step": d2h_total / n_steps,
-            "steps": n_steps, "first_step": first_step, "host_wall_s": wall}
+            "steps": n_steps, "first_step": first_step, "host_wall_s": wall,
+            "host_submit_ms_per_step": 1e3 * submit / n_steps,
+            "h2d_ms_per_step": sum(copy_ms) / n_steps,
+            "h2d_gbs": (h2d_total / 1e9) / (sum(copy_ms) / 1e3) if sum(copy_ms) > 0 else None}
 
 
 # -- budget versus no budget on one session ---------------------------------------------------
@@ -606,7 +635,7 @@ def main():
     out = run_ours(args, rank, world, local_rank)
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:
-            out["cpu_baseline"] = oracle_sample(layers_sampled=2)
+            out["cpu_baseline"] = oracle_sample(layers_sampled=20)
         print(json.dumps(out))
     if world > 1:
         import torch

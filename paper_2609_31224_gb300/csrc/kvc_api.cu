@@ -35,7 +35,7 @@ int fail(int code, const char* fmt, ...) {
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Sizes {
-  int max_moves, max_alloc, dec_slots, max_pf_items;
+  int max_moves, max_alloc, dec_slots, dec_tag_slots, max_pf_items;
 };
 
 Sizes derive_sizes(const kvc_config& c) {
@@ -45,6 +45,8 @@ Sizes derive_sizes(const kvc_config& c) {
   s.max_alloc = s.max_moves / PS + c.max_tokens_per_call / PS + 2 * c.max_seq_per_call + 1;
   // Decode partial slots: two per CTA of the stream-K split (grid <= 2048 CTAs).
   s.dec_slots = 4096;
+  // Tagged partial slots of the pair-split decode (one per CTA of its one-wave grid).
+  s.dec_tag_slots = 2048;
   // Prefill partial slots: the binary32 kernel's chunk list, and two per CTA of the
   // bfloat16 kernel's stream-K split.
   s.max_pf_items = (int)std::min<int64_t>(2048, std::max<int64_t>(512, (int64_t)c.max_seq_per_call * c.kv_heads * 4));
@@ -82,6 +84,7 @@ size_t layout_meta(const kvc_config& c, uint8_t* base, Dev* d) {
   uint8_t* al = take((size_t)z.max_alloc * 4);
   uint8_t* dpo = take((size_t)z.dec_slots * G * c.head_dim * 4);
   uint8_t* dpm = take((size_t)z.dec_slots * G * sizeof(float2));
+  uint8_t* dtg = take((size_t)z.dec_tag_slots * (G * c.head_dim + 2 * G) * 8);
   uint8_t* ppo = take((size_t)z.max_pf_items * PF_MAX_TOKENS * G * 128 * 4);
   uint8_t* ppm = take((size_t)z.max_pf_items * PF_MAX_TOKENS * G * sizeof(float2));
   uint8_t* dc = take((size_t)c.max_seq_per_call * c.kv_heads * 4);
@@ -105,6 +108,8 @@ size_t layout_meta(const kvc_config& c, uint8_t* base, Dev* d) {
     d->alloc_list = reinterpret_cast<int32_t*>(al);
     d->dec_part_o = reinterpret_cast<float*>(dpo);
     d->dec_part_ml = reinterpret_cast<float2*>(dpm);
+    d->dec_tagged = reinterpret_cast<unsigned long long*>(dtg);
+    d->dec_tag_slots = z.dec_tag_slots;
     d->pf_part_o = reinterpret_cast<float*>(ppo);
     d->pf_part_ml = reinterpret_cast<float2*>(ppm);
     d->dec_count = reinterpret_cast<int32_t*>(dc);
@@ -169,6 +174,7 @@ struct kvc_ctx {
   uint64_t layers_written = 0;  // layers whose K/V of the last append are in the pool
   bool last_single = false;
   int pf_target = 0;
+  uint32_t dec_epoch = 0;  // tag of the last decode launch's partial states
 };
 
 namespace {
@@ -188,6 +194,29 @@ int check_sessions(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions) {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// Tag for the next decode launch's partial states, or 0 (fenced arrival) while
+// the stream is being captured: a graph replays a launch with the tag it was
+// captured with, which older words in the slots may carry.  When the counter
+// wraps the slots are cleared first, so no word keeps a tag that comes round again.
+cudaError_t next_decode_epoch(kvc_ctx* ctx, cudaStream_t s, uint32_t* epoch) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(s, &st);
+  if (e != cudaSuccess) return e;
+  if (st != cudaStreamCaptureStatusNone) {
+    *epoch = 0;
+    return cudaSuccess;
+  }
+  if (++ctx->dec_epoch == 0) {
+    const int G = ctx->cfg.q_heads / ctx->cfg.kv_heads;
+    e = cudaMemsetAsync(ctx->d.dec_tagged, 0,
+                        (size_t)ctx->d.dec_tag_slots * (G * ctx->cfg.head_dim + 2 * G) * 8, s);
+    if (e != cudaSuccess) return e;
+    ctx->dec_epoch = 1;
+  }
+  *epoch = ctx->dec_epoch;
+  return cudaSuccess;
+}
 
 void enqueue_readback(kvc_ctx* ctx, cudaStream_t s) {
   cudaMemcpyAsync(ctx->h_readback, &ctx->d.g->pages_used, sizeof(int64_t), cudaMemcpyDeviceToHost,
@@ -431,8 +460,11 @@ int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void*
     return fail(KVC_ESTATE, "decode needs exactly one appended token per session");
   // The first attention launch after an append follows the kernel that wrote the
   // new token's K/V, so it does not start early; later ones may.
+  uint32_t epoch = 0;
+  KVC_CUDA(next_decode_epoch(ctx, static_cast<cudaStream_t>(stream), &epoch));
   KVC_CUDA(launch_attn_decode(ctx->d, layer, d_q, d_out, ctx->last_n_seq,
-                              ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream)));
+                              ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream),
+                              epoch));
   ++ctx->attn_since_append;
   return KVC_OK;
 }
@@ -448,9 +480,11 @@ int kvc_attn_decode_kv(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v
     return fail(KVC_ESTATE, "decode needs exactly one appended token per session");
   // Launches after the append may start early: the new rows go into the tiles
   // after their loads, and the previous launch writes another layer's rows only.
+  uint32_t epoch = 0;
+  KVC_CUDA(next_decode_epoch(ctx, static_cast<cudaStream_t>(stream), &epoch));
   KVC_CUDA(launch_attn_decode(ctx->d, layer, d_q, d_out, ctx->last_n_seq,
-                              ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream), d_k,
-                              d_v));
+                              ctx->attn_since_append > 0, static_cast<cudaStream_t>(stream),
+                              epoch, d_k, d_v));
   ctx->layers_written |= 1ull << layer;
   ++ctx->attn_since_append;
   return KVC_OK;

@@ -15,7 +15,12 @@
 //     k slices, one per CTA of 16 warps (one CTA per SM), so that every page of
 //     the call is in flight at once.
 // Either way partial states go to global slots and the last CTA to arrive for a
-// pair merges them (log-sum-exp).
+// pair merges them (log-sum-exp).  Stream-K publishes them with an acquire-release
+// arrival.  The 16-warp pair split, whose launches are latency-bound, writes each
+// partial value as a word tagged with the launch and arrives with a relaxed atomic,
+// so no release fence sits on its critical path; the merging CTA re-reads the words
+// whose tag is not yet current.  Launches captured into a graph (where a replay
+// would repeat the tag) use the acquire-release arrival.
 #include "kvc_internal.cuh"
 
 namespace kvc {
@@ -532,6 +537,109 @@ __device__ void merge_parts(const Dev& d, const Smem<C>& sm, int nch, PartFn par
   }
 }
 
+// Tagged partial state of slot `slot`: G * D output words, then (m, l) per row.
+template <class C>
+__device__ inline unsigned long long* tagged_slot(const Dev& d, int slot) {
+  return d.dec_tagged + (size_t)slot * (G * C::D + 2 * G);
+}
+
+// Write this CTA's merged warps (merge_warps done) as the tagged partial state of
+// `slot`.  Called by every thread.
+template <class C>
+__device__ void publish_tagged(const Dev& d, const Smem<C>& sm, int slot, uint32_t tag,
+                               int tid) {
+  unsigned long long* ts = tagged_slot<C>(d, slot);
+  for (int e = tid; e < G * C::D; e += C::THREADS) st_tagged(ts + e, tag, merge_warps_elem<C>(sm, e));
+  if (tid < 2 * G) st_tagged(ts + G * C::D + tid, tag, sm.r_ml[tid]);
+}
+
+// merge_parts over the tagged states of slots slot0 .. slot0 + nch - 1 of this
+// launch (tag): every load is a single 64-bit word whose tag says whether its
+// store has landed.
+template <class C>
+__device__ void merge_tagged(const Dev& d, const Smem<C>& sm, int nch, int slot0, uint32_t tag,
+                             typename C::T* orow, int tid, int warp, int lane) {
+  using T = typename C::T;
+  constexpr int D = C::D, TW = G * D + 2 * G;
+  static_assert(C::WARPS >= G, "one warp per query row");
+  constexpr int EPT = (G * D + C::THREADS - 1) / C::THREADS;
+  constexpr int CH = 24 / EPT > 0 ? 24 / EPT : 1;
+  const unsigned long long* base = tagged_slot<C>(d, slot0);
+  const unsigned long long filler = (unsigned long long)tag << 32;  // 0.0f, current tag
+  unsigned long long a[CH][EPT];
+  auto load_batch = [&](int c0) {
+#pragma unroll
+    for (int i = 0; i < CH; ++i)
+#pragma unroll
+      for (int t = 0; t < EPT; ++t) {
+        const int e = tid + t * C::THREADS;
+        a[i][t] = (c0 + i < nch && e < G * D) ? ld_tagged(base + (size_t)(c0 + i) * TW + e)
+                                              : filler;
+      }
+  };
+  load_batch(0);
+  if (warp < G) {
+    const int g = warp;
+    constexpr int PL = MAX_PARTS / 32;
+    unsigned long long wm[PL], wl[PL];
+#pragma unroll
+    for (int i = 0; i < PL; ++i) {
+      const int ch = lane + 32 * i;
+      const unsigned long long* p = base + (size_t)ch * TW + G * D + 2 * g;
+      wm[i] = ch < nch ? ld_tagged(p) : filler;
+      wl[i] = ch < nch ? ld_tagged(p + 1) : filler;
+    }
+    float m[PL], l[PL], M = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < PL; ++i) {
+      const int ch = lane + 32 * i;
+      const unsigned long long* p = base + (size_t)ch * TW + G * D + 2 * g;
+      m[i] = ch < nch ? tagged_value(d, p, wm[i], tag) : -INFINITY;
+      l[i] = ch < nch ? tagged_value(d, p + 1, wl[i], tag) : 0.f;
+      M = fmaxf(M, m[i]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(FULL, M, o));
+    float sc[PL], L = 0.f;
+#pragma unroll
+    for (int i = 0; i < PL; ++i) {
+      sc[i] = exp2_safe(m[i], M);
+      L += l[i] * sc[i];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(FULL, L, o);
+    const float inv = 1.f / L;
+#pragma unroll
+    for (int i = 0; i < PL; ++i)
+      if (lane + 32 * i < nch) sm.s_scale[(lane + 32 * i) * G + g] = sc[i] * inv;
+  }
+  __syncthreads();
+  float O[EPT];
+#pragma unroll
+  for (int t = 0; t < EPT; ++t) O[t] = 0.f;
+  for (int c0 = 0;;) {
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      if (c0 + i >= nch) break;
+#pragma unroll
+      for (int t = 0; t < EPT; ++t) {
+        const int e = tid + t * C::THREADS;
+        if (e < G * D)
+          O[t] += tagged_value(d, base + (size_t)(c0 + i) * TW + e, a[i][t], tag) *
+                  sm.s_scale[(c0 + i) * G + e / D];
+      }
+    }
+    c0 += CH;
+    if (c0 >= nch) break;
+    load_batch(c0);
+  }
+#pragma unroll
+  for (int t = 0; t < EPT; ++t) {
+    const int e = tid + t * C::THREADS;
+    if (e < G * D) orow[e] = from_float<T>(O[t]);
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Stream-K kernel.
 // ---------------------------------------------------------------------------
@@ -644,7 +752,7 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
 template <typename T, int D, bool FUSED, class C>
 __global__ void __launch_bounds__(C::THREADS) attn_decode_split_kernel(
     Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale, int k,
-    const T* new_k, const T* new_v) {
+    uint32_t epoch, const T* new_k, const T* new_v) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const Smem<C> sm(smem, warp);
@@ -686,6 +794,16 @@ __global__ void __launch_bounds__(C::THREADS) attn_decode_split_kernel(
   merge_warps<C>(sm, warp, lane);
   T* orow = out + ((size_t)si.q_row0 * d.q_heads + head * G) * D;
   const int slot = blockIdx.x;
+  if (k > 1 && epoch != 0) {
+    publish_tagged<C>(d, sm, slot, epoch, tid);
+    __syncthreads();
+    if (tid == 0) s_last = arrive_relaxed(&d.dec_count[pair], k);
+    __syncthreads();
+    if (!s_last) return;
+    merge_tagged<C>(d, sm, k, pair * k, epoch, orow, tid, warp, lane);
+    if (tid == 0) d.dec_count[pair] = 0;
+    return;
+  }
   for (int e = tid; e < G * D; e += C::THREADS) {
     const float O = merge_warps_elem<C>(sm, e);
     const int g = e / D;
@@ -740,12 +858,13 @@ int split_slots() {
 constexpr int DEC_MIN_UNITS = 12;
 // The pair-split kernel takes calls whose pairs each get at least this many CTAs
 // in one wave: with 16-warp CTAs (one per SM) first, else with stream-K's 4-warp
-// CTAs (three per SM).
+// CTAs (three per SM).  Only the 16-warp shape uses tagged partial states: with
+// 4-warp CTAs the fenced arrival measured faster.
 constexpr int SPLIT_MIN_K = 2, SPLIT4_MIN_K = 3;
 
 template <typename T, int D>
 cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int n_seq, bool pdl,
-                          cudaStream_t s, const void* new_k, const void* new_v) {
+                          cudaStream_t s, uint32_t epoch, const void* new_k, const void* new_v) {
   static thread_local const int grid = stream_k_grid<T, D>(d);
   static thread_local const int slots = split_slots<T, D, SpCfg<T, D>>();
   static thread_local const int slots4 = split_slots<T, D, SkCfg<T, D>>();
@@ -762,7 +881,7 @@ cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int
     return launch_ex(fused ? &attn_decode_split_kernel<T, D, true, C>
                            : &attn_decode_split_kernel<T, D, false, C>,
                      dim3(n_pairs * k), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, qt, ot,
-                     scale, k, nk, nv);
+                     scale, k, n_pairs * k <= d.dec_tag_slots ? epoch : 0u, nk, nv);
   }
   const int k4 = n_pairs * SPLIT4_MIN_K <= slots4 ? min(MAX_PARTS, slots4 / n_pairs) : 0;
   if (k4 > 0) {
@@ -770,7 +889,7 @@ cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int
     return launch_ex(fused ? &attn_decode_split_kernel<T, D, true, C>
                            : &attn_decode_split_kernel<T, D, false, C>,
                      dim3(n_pairs * k4), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, qt, ot,
-                     scale, k4, nk, nv);
+                     scale, k4, 0u, nk, nv);
   }
   return launch_ex(fused ? &attn_decode_kernel<T, D, true> : &attn_decode_kernel<T, D, false>,
                    dim3(grid), dim3(SkCfg<T, D>::THREADS), SkCfg<T, D>::SMEM, s, pdl, d, layer,
@@ -780,10 +899,12 @@ cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int
 }  // namespace
 
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               bool pdl, cudaStream_t s, const void* new_k, const void* new_v) {
+                               bool pdl, cudaStream_t s, uint32_t epoch, const void* new_k,
+                               const void* new_v) {
   if (d.esz == 2)
-    return launch_decode<__nv_bfloat16, 128>(d, layer, q, out, n_seq, pdl, s, new_k, new_v);
-  return launch_decode<float, 64>(d, layer, q, out, n_seq, pdl, s, new_k, new_v);
+    return launch_decode<__nv_bfloat16, 128>(d, layer, q, out, n_seq, pdl, s, epoch, new_k,
+                                             new_v);
+  return launch_decode<float, 64>(d, layer, q, out, n_seq, pdl, s, epoch, new_k, new_v);
 }
 
 }  // namespace kvc

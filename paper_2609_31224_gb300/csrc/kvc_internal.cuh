@@ -107,6 +107,8 @@ struct Dev {
   int32_t max_alloc;
   float* dec_part_o;           // [dec_slots][G][D]
   float2* dec_part_ml;         // [dec_slots][G] (m, l) in log2 units
+  unsigned long long* dec_tagged;  // [dec_tag_slots][G * D + 2 G] tagged partial states
+  int32_t dec_tag_slots;
   float* pf_part_o;            // [max_pf_items][PF_ROWS][D]
   float2* pf_part_ml;          // [max_pf_items][PF_ROWS]
   int32_t* dec_count;          // [max_seq * kv_heads] arrival counters
@@ -246,6 +248,43 @@ __device__ inline int block_page(const SeqInfo& si, const int32_t* hist_row,
 }
 
 __device__ inline void set_error(const Dev& d, int bits) { atomicOr(&d.g->err, bits); }
+
+// Tagged partial states.  A CTA writes each value of its partial state as one
+// 64-bit word, (tag << 32) | binary32 bits, and arrives with a relaxed atomic: no
+// release fence waits for its stores.  The last CTA to arrive reads each word
+// with a single-copy-atomic 64-bit load and re-reads (bounded) any word whose tag
+// is not yet the launch's: the stores it waits for were issued before their CTAs'
+// arrivals, so the wait needs no other CTA to make progress.
+__device__ inline void st_tagged(unsigned long long* p, uint32_t tag, float v) {
+  const unsigned long long w = ((unsigned long long)tag << 32) | __float_as_uint(v);
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(w) : "memory");
+}
+__device__ inline unsigned long long ld_tagged(const unsigned long long* p) {
+  unsigned long long w;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
+  return w;
+}
+// Value of word w (loaded from p) once its tag is `tag`; 0 with KVC_DERR_WAIT
+// recorded if the store does not show up within WAIT_LIMIT_CYCLES.
+__device__ inline float tagged_value(const Dev& d, const unsigned long long* p,
+                                     unsigned long long w, uint32_t tag) {
+  if ((uint32_t)(w >> 32) != tag) {
+    const long long t0 = clock64();
+    do {
+      if (clock64() - t0 > WAIT_LIMIT_CYCLES) {
+        set_error(d, KVC_DERR_WAIT);
+        return 0.f;
+      }
+      w = ld_tagged(p);
+    } while ((uint32_t)(w >> 32) != tag);
+  }
+  return __uint_as_float((uint32_t)w);
+}
+__device__ inline bool arrive_relaxed(int* counter, int parts) {
+  int old;
+  asm volatile("atom.relaxed.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(counter) : "memory");
+  return old == parts - 1;
+}
 
 // ---------------------------------------------------------------------------
 // PTX helpers: mbarrier and bulk (TMA) copies global -> shared.
@@ -405,9 +444,11 @@ cudaError_t launch_release(const Dev& d, const SeqArgs& a, cudaStream_t s);
 cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_out, void* k_out,
                               void* v_out, int32_t* count, cudaStream_t s);
 // new_k / new_v (optional): the fused per-layer write of the new tokens' K/V.
+// epoch: tag of this launch's partial states (nonzero, never reused while tags
+// of it may remain in the slots); 0 selects the fenced arrival instead.
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               bool pdl, cudaStream_t s, const void* new_k = nullptr,
-                               const void* new_v = nullptr);
+                               bool pdl, cudaStream_t s, uint32_t epoch,
+                               const void* new_k = nullptr, const void* new_v = nullptr);
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                 int max_t, bool pdl, cudaStream_t s);
 cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,

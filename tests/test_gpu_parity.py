@@ -400,3 +400,43 @@ def test_error_codes():
     c.release([0])
     free, err = c.device_status()
     assert free == 3
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_decode_graph_replay_matches_eager(dtype):
+    """Decode launches captured in a CUDA graph merge their split-K partial states after
+    a fenced arrival (a replay repeats the captured arguments); eager launches tag each
+    partial word with the launch.  Both merge in the same order, so the outputs are
+    bit-identical, across replays and for eager launches after them."""
+    w = S.SINGLE_BF16.with_(layers=2, n_sessions=12, units=80, seed=5)
+    if dtype == "f32":
+        w = w.with_(dtype="f32", head_dim=64)
+    drv = Driver(w, S.workload_scripts(w))
+    drv.fast_forward(60)
+    torch.cuda.synchronize()
+    for n in (1, 4, 12):
+        c = drv._make_call("decode", list(range(n)), [np.array([3], np.uint8)] * n, True)
+        drv.cache.append_chunk(c.sessions, c.cu, c.types, c.k, c.v)
+        eager = []
+        for layer in range(w.layers):
+            drv.cache.attn_decode(layer, c.q[layer], c.out)
+            eager.append(c.out.clone())
+        outs = [torch.empty_like(c.out) for _ in range(w.layers)]
+        g = torch.cuda.CUDAGraph()
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.graph(g, stream=s):
+            for layer in range(w.layers):
+                drv.cache.attn_decode(layer, c.q[layer], outs[layer], stream=s)
+        for _ in range(3):
+            for o in outs:
+                o.zero_()
+            g.replay()
+            torch.cuda.synchronize()
+            for layer in range(w.layers):
+                assert torch.equal(outs[layer], eager[layer]), (n, layer)
+        for layer in range(w.layers):
+            drv.cache.attn_decode(layer, c.q[layer], c.out)
+            assert torch.equal(c.out, eager[layer]), (n, layer)
+        del g
+        torch.cuda.synchronize()
