@@ -21,6 +21,8 @@
 // so no release fence sits on its critical path; the merging CTA re-reads the words
 // whose tag is not yet current.  Launches captured into a graph (where a replay
 // would repeat the tag) use the acquire-release arrival.
+#include <cstring>
+
 #include "kvc_internal.cuh"
 
 namespace kvc {
@@ -33,28 +35,32 @@ constexpr float LOG2E = 1.4426950408889634f;
 constexpr int MAX_PARTS = 64;     // partial states per (session, head) pair, at most
 
 // One CTA shape: WARPS warps, each streaming its own pages through a STAGES-deep
-// ring of K/V tiles.
-template <typename T_, int D_, int WARPS_, int STAGES_>
+// ring of K/V tiles.  MMA (bfloat16 only): the page loop runs on the tensor cores
+// (mma.sync), with tiles staged by 2-D TMA in the 128-byte-swizzled layout;
+// otherwise on CUDA cores with tiles staged by 1-D bulk copies.
+template <typename T_, int D_, int WARPS_, int STAGES_, bool MMA_ = false>
 struct DecCfg {
   using T = T_;
   static constexpr int D = D_, WARPS = WARPS_, STAGES = STAGES_, THREADS = WARPS * 32;
   static constexpr int ESZ = sizeof(T);
+  static constexpr bool MMA = MMA_ && ESZ == 2;
   static constexpr int ROW_BYTES = D * ESZ;
   static_assert(ROW_BYTES == 256, "decode kernel assumes 256-byte K/V rows");
   static constexpr int VEC = 16 / ESZ;     // elements per 16-byte lane chunk (QK)
   static constexpr int PVD = D / 32;       // dims per lane (PV)
   static constexpr int TILE = PS * ROW_BYTES;  // one page of one head: 4 KiB
-  // shared memory per warp: STAGES x (K tile + V tile) + scores + probability
-  // pairs (p, p) + alpha
-  static constexpr int WARP_BYTES = STAGES * 2 * TILE + (G * PS + 2 * PS * G + G) * 4 + 16;
-  static_assert(WARP_BYTES % 16 == 0, "bulk-copy destinations must stay 16-byte aligned");
+  // Shared memory (from a 1024-aligned base): every warp's STAGES x (K tile + V
+  // tile), then per warp: scores + probability pairs (p, p) + alpha.
+  static constexpr int TILES = WARPS * STAGES * 2 * TILE;
+  static constexpr int SCRATCH = (G * PS + 2 * PS * G + G) * 4 + 16;
+  static_assert(SCRATCH % 16 == 0, "scratch stays 16-byte aligned");
   // The cross-warp merge reuses the stage buffers once every warp is done with
   // its pages.
   static constexpr int MERGE_FLOATS = WARPS * G * D + WARPS * G * 2;
   static constexpr int RESULT_FLOATS = G * 2 + WARPS * G;
-  static_assert((MERGE_FLOATS + RESULT_FLOATS) * 4 <= WARPS * WARP_BYTES,
-                "merge area must fit in the stages");
-  static constexpr int SMEM = WARPS * WARP_BYTES + WARPS * STAGES * 8 + MAX_PARTS * G * 4 + 64;
+  static_assert((MERGE_FLOATS + RESULT_FLOATS) * 4 <= TILES, "merge area must fit in the stages");
+  static constexpr int SMEM =
+      1024 + TILES + WARPS * SCRATCH + WARPS * STAGES * 8 + MAX_PARTS * G * 4 + 64;
 };
 
 // Stream-K kernel: 4 warps (one per query row in the split-K merge), 2-deep rings,
@@ -62,10 +68,15 @@ struct DecCfg {
 template <typename T, int D>
 using SkCfg = DecCfg<T, D, 4, 2>;
 // Pair-split kernel: 16 warps, one tile pair each, one CTA per SM; with few
-// sessions every page of the call is in flight at once.
+// sessions every page of the call is in flight at once.  Its pages are latency-
+// bound, so for bfloat16 they run on the tensor cores (fewer instructions per page).
 constexpr int SP_WARPS = 16, SP_STAGES = 1;
 template <typename T, int D>
-using SpCfg = DecCfg<T, D, SP_WARPS, SP_STAGES>;
+using SpCfg = DecCfg<T, D, SP_WARPS, SP_STAGES, true>;
+// Pair-split kernel for calls with too many pairs for SpCfg: stream-K's CTA shape.
+constexpr bool SP4_MMA = false;
+template <typename T, int D>
+using Sp4Cfg = DecCfg<T, D, 4, 2, SP4_MMA>;
 
 template <typename T>
 __device__ inline void load_vec(const uint8_t* p, float* f);
@@ -107,17 +118,21 @@ struct Smem {
   float* s_wsc;       // [W][G] weight of each warp's part (aliases the stages)
   uint64_t* wbars;    // this warp's [STAGES]
   float* s_scale;     // [MAX_PARTS][G]
-  __device__ Smem(uint8_t* smem, int warp) {
-    uint8_t* wbase = smem + warp * C::WARP_BYTES;
-    tiles = wbase;
-    s_sc = reinterpret_cast<float*>(wbase + C::STAGES * 2 * C::TILE);
+  // The tensor-core page loop keeps the bfloat16 probabilities P^T [G rows][PS
+  // keys] in s_sc.
+  __device__ Smem(uint8_t* raw, int warp) {
+    // Offset into the shared array itself (keeps the accesses shared-memory ones).
+    uint8_t* smem = raw + ((1024u - (smem_u32(raw) & 1023u)) & 1023u);
+    tiles = smem + warp * C::STAGES * 2 * C::TILE;
+    uint8_t* scratch = smem + C::TILES + warp * C::SCRATCH;
+    s_sc = reinterpret_cast<float*>(scratch);
     s_p2 = reinterpret_cast<float2*>(s_sc + G * PS);
     s_alpha = reinterpret_cast<float*>(s_p2 + PS * G);
     m_o = reinterpret_cast<float*>(smem);
     m_ml = m_o + C::WARPS * G * C::D;
     r_ml = m_ml + C::WARPS * G * 2;
     s_wsc = r_ml + G * 2;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::WARPS * C::WARP_BYTES);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::TILES + C::WARPS * C::SCRATCH);
     wbars = bars + warp * C::STAGES;
     s_scale = reinterpret_cast<float*>(bars + C::WARPS * C::STAGES);
   }
@@ -135,8 +150,13 @@ struct Segment {
   const int32_t* hrow;
   const int32_t* lrow;
   int pwin, pid;
+  const CUtensorMap* map_lo;  // tensor maps of the pool (tensor-core page loop only)
+  const CUtensorMap* map_hi;
 
-  __device__ void init(const Dev& d, const SeqInfo& s, int h, int b0, int nb, int warp) {
+  __device__ void init(const Dev& d, const SeqInfo& s, int h, int b0, int nb, int warp,
+                       const CUtensorMap* mlo = nullptr, const CUtensorMap* mhi = nullptr) {
+    map_lo = mlo;
+    map_hi = mhi;
     si = s;
     head = h;
     blk_begin = b0;
@@ -161,11 +181,21 @@ struct Segment {
       const uint32_t n = loads + k;
       const int st = n % C::STAGES;
       uint8_t* dst = sm.tiles + st * 2 * C::TILE;
-      const T* kp = reinterpret_cast<const T*>(d.pool) +
-                    pool_offset_elems(d, page, layer, 0, head, 0);
       mbar_arrive_expect_tx(&sm.wbars[st], 2 * C::TILE);
-      bulk_g2s(dst, kp, C::TILE, &sm.wbars[st]);
-      bulk_g2s(dst + C::TILE, kp + (size_t)d.kv_heads * PS * D, C::TILE, &sm.wbars[st]);
+      if constexpr (C::MMA) {
+        // Pool rows of the K and V tiles, each as two swizzled 64-column boxes.
+        const int krow = (((page * d.layers + layer) * 2) * d.kv_heads + head) * PS;
+        const int vrow = krow + d.kv_heads * PS;
+        tma_load_2d(dst, map_lo, 0, krow, &sm.wbars[st]);
+        tma_load_2d(dst + C::TILE / 2, map_hi, 0, krow, &sm.wbars[st]);
+        tma_load_2d(dst + C::TILE, map_lo, 0, vrow, &sm.wbars[st]);
+        tma_load_2d(dst + C::TILE + C::TILE / 2, map_hi, 0, vrow, &sm.wbars[st]);
+      } else {
+        const T* kp = reinterpret_cast<const T*>(d.pool) +
+                      pool_offset_elems(d, page, layer, 0, head, 0);
+        bulk_g2s(dst, kp, C::TILE, &sm.wbars[st]);
+        bulk_g2s(dst + C::TILE, kp + (size_t)d.kv_heads * PS * D, C::TILE, &sm.wbars[st]);
+      }
     }
   }
 
@@ -224,21 +254,28 @@ __device__ void patch_new_row(const Dev& d, int layer, const SeqInfo& si, int he
   const float2* cs = d.rope + (size_t)si.pos_first * HALF;
   T* kp = reinterpret_cast<T*>(d.pool) + pool_offset_elems(d, page, layer, 0, head, slot);
   T* vp = reinterpret_cast<T*>(d.pool) + pool_offset_elems(d, page, layer, 1, head, slot);
-  T* kr = reinterpret_cast<T*>(kt + slot * C::ROW_BYTES);
-  T* vr = reinterpret_cast<T*>(kt + C::TILE + slot * C::ROW_BYTES);
+  // Byte offset of element j of the row within a tile (linear, or two swizzled
+  // 64-column boxes for the tensor-core loop).
+  auto at = [&](int j) -> int {
+    if constexpr (C::MMA)
+      return (j >> 6) * (C::TILE / 2) + slot * 128 + ((((j & 63) >> 3) ^ (slot & 7)) << 4) +
+             (j & 7) * C::ESZ;
+    else
+      return slot * C::ROW_BYTES + j * C::ESZ;
+  };
   for (int j = lane; j < HALF; j += 32) {
     const float x1 = to_float<T>(kin[j]), x2 = to_float<T>(kin[j + HALF]);
     const float2 c = cs[j];
     const T y1 = from_float<T>(fmaf(x1, c.x, -x2 * c.y));
     const T y2 = from_float<T>(fmaf(x2, c.x, x1 * c.y));
-    kr[j] = y1;
-    kr[j + HALF] = y2;
+    *reinterpret_cast<T*>(kt + at(j)) = y1;
+    *reinterpret_cast<T*>(kt + at(j + HALF)) = y2;
     kp[j] = y1;
     kp[j + HALF] = y2;
   }
   for (int j = lane; j < D; j += 32) {
     const T x = vin[j];
-    vr[j] = x;
+    *reinterpret_cast<T*>(kt + C::TILE + at(j)) = x;
     vp[j] = x;
   }
   __syncwarp();
@@ -361,6 +398,219 @@ __device__ int stream_pages(const Dev& d, int layer, Segment<C>& sg, const Smem<
     }
   }
   return -1;
+}
+
+// ---------------------------------------------------------------------------
+// Tensor-core page loop (bfloat16, D = 128).  Per page of 16 keys and the G = 4
+// query rows of one KV head, with the keys as the MMA's M dimension:
+//   S^T [16 keys x 8 rows]  = K [16 x 128] . Q^T [128 x 8]        (8 k-steps)
+//   O^T [128 dims x 8 rows] += V^T [128 x 16 keys] . P^T [16 x 8]  (8 m-tiles)
+// with mma.sync m16n8k16 (bf16 in, fp32 accumulate); rows 4..7 are zero padding.
+// Lane (g, t) = (lane >> 2, lane & 3) holds S^T for keys g, g + 8 and rows 2t,
+// 2t + 1, so it owns the softmax state of rows 2t, 2t + 1 (valid for t < 2), and
+// O^T for dims 16 mt + g (+ 8) of the same rows.  Tiles are two 64-column boxes
+// (2 KiB, 16 rows of 128 B) with the 128-byte swizzle: 16-byte chunk c of row r
+// sits at chunk c ^ (r & 7), so ldmatrix reads of 8 rows hit 8 distinct banks.
+// ---------------------------------------------------------------------------
+__device__ inline uint32_t swz(int row, int col) {  // col: a multiple of 8 in [0, 128)
+  return (col >> 6) * 2048 + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4);
+}
+
+__device__ inline void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ inline void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ inline void mma_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                 uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ inline uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// Query rows of `head`, rotated at the token's position, scaled by log2(e)/sqrt(D)
+// and rounded to bfloat16, as the B operand Q^T of the score products: lane (g, t)
+// with g < G holds dims 16 ks + 2t, +1 (qb[ks][0]) and 16 ks + 2t + 8, +9
+// (qb[ks][1]) of row g; lanes g >= G hold the zero rows.  Dims d and d + 64 (k-steps
+// ks and ks + 4 of the same lane) are rotated together.
+template <class C>
+__device__ void load_q_mma(const Dev& d, const SeqInfo& si, int head, const typename C::T* q,
+                           float qk_scale, int lane, uint32_t (&qb)[8][2]) {
+  static_assert(C::D == 128, "tensor-core page loop assumes D = 128");
+  const int g = lane >> 2, t = lane & 3;
+  if (g >= G) {
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) qb[ks][0] = qb[ks][1] = 0u;
+    return;
+  }
+  const uint32_t* qrow = reinterpret_cast<const uint32_t*>(
+      q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G + g) * C::D);
+  const float2* cs = d.rope + (size_t)si.pos_first * (C::D / 2);
+  uint32_t w[8][2];
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    w[ks][0] = qrow[8 * ks + t];
+    w[ks][1] = qrow[8 * ks + t + 4];
+  }
+  float2 c[4][4];
+#pragma unroll
+  for (int ks = 0; ks < 4; ++ks)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      c[ks][2 * j] = cs[16 * ks + 2 * t + 8 * j];
+      c[ks][2 * j + 1] = cs[16 * ks + 2 * t + 8 * j + 1];
+    }
+#pragma unroll
+  for (int ks = 0; ks < 4; ++ks)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const float x0 = bf16lo(w[ks][j]), x1 = bf16hi(w[ks][j]);          // dims < 64
+      const float y0 = bf16lo(w[ks + 4][j]), y1 = bf16hi(w[ks + 4][j]);  // dims + 64
+      const float2 c0 = c[ks][2 * j], c1 = c[ks][2 * j + 1];
+      qb[ks][j] = pack_bf16x2(fmaf(x0, c0.x, -y0 * c0.y) * qk_scale,
+                              fmaf(x1, c1.x, -y1 * c1.y) * qk_scale);
+      qb[ks + 4][j] = pack_bf16x2(fmaf(y0, c0.x, x0 * c0.y) * qk_scale,
+                                  fmaf(y1, c1.x, x1 * c1.y) * qk_scale);
+    }
+}
+
+// stream_pages on the tensor cores.  m_run / l_run: running max and this lane's
+// partial sum of rows 2t, 2t + 1 (the sum is completed over g by publish_warp_mma).
+template <class C, bool FUSED>
+__device__ int stream_pages_mma(const Dev& d, int layer, Segment<C>& sg, const Smem<C>& sm,
+                                uint32_t loads, const uint32_t (&qb)[8][2], float (&m_run)[2],
+                                float (&l_run)[2], float (&o)[8][4], int warp, int lane,
+                                const typename C::T* new_k, const typename C::T* new_v) {
+  const int g = lane >> 2, t = lane & 3;
+  // ldmatrix row of this lane: K (A = K, keys x dims) and V (A = V^T via .trans).
+  const int k_key = (lane & 7) + 8 * ((lane >> 3) & 1), k_col = 8 * (lane >> 4);
+  const int v_key = (lane & 7) + 8 * (lane >> 4), v_col = 8 * ((lane >> 3) & 1);
+  __nv_bfloat16* pt = reinterpret_cast<__nv_bfloat16*>(sm.s_sc);  // P^T as [G][PS]
+  for (int k = 0; k < sg.n_my; ++k) {
+    const uint32_t n = loads + k;
+    const int st = n % C::STAGES;
+    if (!__all_sync(FULL, mbar_wait(d, &sm.wbars[st], (n / C::STAGES) & 1))) return k;
+    uint8_t* kt = sm.tiles + st * 2 * C::TILE;
+    const int blk = sg.blk_begin + warp + k * C::WARPS;
+    if constexpr (FUSED) {
+      if (blk == sg.si.n_blocks - 1)
+        patch_new_row<C>(d, layer, sg.si, sg.head, new_k, new_v, kt, lane);
+    }
+    const uint32_t kb = smem_u32(kt), vb = kb + C::TILE;
+
+    float s[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      uint32_t a[4];
+      ldsm_x4(a, kb + swz(k_key, 16 * ks + k_col));
+      mma_16816(s, a, qb[ks][0], qb[ks][1]);
+    }
+    const BlockRange br = block_range(sg.si, blk);
+    if (!(br.lo == 0 && br.hi == PS)) {
+      if (g < br.lo || g >= br.hi) s[0] = s[1] = -INFINITY;
+      if (g + 8 < br.lo || g + 8 >= br.hi) s[2] = s[3] = -INFINITY;
+    }
+    // Online softmax of rows 2t (s0, s2) and 2t + 1 (s1, s3) over the page's keys.
+    float mx0 = fmaxf(s[0], s[2]), mx1 = fmaxf(s[1], s[3]);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      mx0 = fmaxf(mx0, __shfl_xor_sync(FULL, mx0, off));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(FULL, mx1, off));
+    }
+    const float mn0 = fmaxf(m_run[0], mx0), mn1 = fmaxf(m_run[1], mx1);
+    const float p0 = exp2_safe(s[0], mn0), p2 = exp2_safe(s[2], mn0);
+    const float p1 = exp2_safe(s[1], mn1), p3 = exp2_safe(s[3], mn1);
+    const float al0 = exp2_safe(m_run[0], mn0), al1 = exp2_safe(m_run[1], mn1);
+    l_run[0] = l_run[0] * al0 + (p0 + p2);
+    l_run[1] = l_run[1] * al1 + (p1 + p3);
+    m_run[0] = mn0;
+    m_run[1] = mn1;
+    // P^T to the B-operand layout through shared memory: lane (g, t < 2) writes
+    // P[row][key] for its two rows and keys g, g + 8; lane (g < G, t) reads keys
+    // 2t, 2t + 1 and 2t + 8, 2t + 9 of row g.
+    __syncwarp();
+    if (t < 2) {
+      pt[(2 * t) * PS + g] = __float2bfloat16_rn(p0);
+      pt[(2 * t + 1) * PS + g] = __float2bfloat16_rn(p1);
+      pt[(2 * t) * PS + g + 8] = __float2bfloat16_rn(p2);
+      pt[(2 * t + 1) * PS + g + 8] = __float2bfloat16_rn(p3);
+    }
+    __syncwarp();
+    uint32_t pb0 = 0u, pb1 = 0u;
+    if (g < G) {
+      pb0 = *reinterpret_cast<const uint32_t*>(pt + g * PS + 2 * t);
+      pb1 = *reinterpret_cast<const uint32_t*>(pt + g * PS + 2 * t + 8);
+    }
+    if (__any_sync(FULL, al0 != 1.f || al1 != 1.f)) {
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        o[mt][0] *= al0;
+        o[mt][1] *= al1;
+        o[mt][2] *= al0;
+        o[mt][3] *= al1;
+      }
+    }
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      uint32_t a[4];
+      ldsm_x4_trans(a, vb + swz(v_key, 16 * mt + v_col));
+      mma_16816(o[mt], a, pb0, pb1);
+    }
+    __syncwarp();
+    if (k + C::STAGES < sg.n_my) {
+      if (lane == 0) fence_proxy_async_smem();
+      sg.issue(d, layer, sm, loads, k + C::STAGES, warp, lane);
+    }
+  }
+  return -1;
+}
+
+// publish_warp for the tensor-core state: completes each row's sum over the lanes
+// holding its keys and writes (m, l) and the row's unnormalised output.
+template <class C>
+__device__ void publish_warp_mma(const Smem<C>& sm, const float (&m_run)[2],
+                                 const float (&l_run)[2], const float (&o)[8][4], int warp,
+                                 int lane) {
+  constexpr int D = C::D;
+  const int g = lane >> 2, t = lane & 3;
+  float l0 = l_run[0], l1 = l_run[1];
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    l0 += __shfl_xor_sync(FULL, l0, off);
+    l1 += __shfl_xor_sync(FULL, l1, off);
+  }
+  if (t < 2) {
+    const int r0 = warp * G + 2 * t, r1 = r0 + 1;
+    if (g == 0) {
+      sm.m_ml[r0 * 2 + 0] = m_run[0];
+      sm.m_ml[r0 * 2 + 1] = l0;
+      sm.m_ml[r1 * 2 + 0] = m_run[1];
+      sm.m_ml[r1 * 2 + 1] = l1;
+    }
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      sm.m_o[r0 * D + 16 * mt + g] = o[mt][0];
+      sm.m_o[r1 * D + 16 * mt + g] = o[mt][1];
+      sm.m_o[r0 * D + 16 * mt + g + 8] = o[mt][2];
+      sm.m_o[r1 * D + 16 * mt + g + 8] = o[mt][3];
+    }
+  }
 }
 
 // After every warp of the CTA has finished (caller syncs): publish the warps'
@@ -640,14 +890,27 @@ __device__ void merge_tagged(const Dev& d, const Smem<C>& sm, int nch, int slot0
   }
 }
 
+// A wait of this warp's page loop gave up at page failed_at (error recorded):
+// drain the copies it still has in flight (bounded waits).  Pair-split layout
+// (loads start at 0).
+template <class C>
+__device__ inline void drain_after_failure(const Dev& d, const Smem<C>& sm, const Segment<C>& sg,
+                                           int failed_at) {
+  if (failed_at < 0) return;
+  for (int j = failed_at; j < min(sg.n_my, failed_at + C::STAGES); ++j)
+    mbar_wait(d, &sm.wbars[j % C::STAGES], (j / C::STAGES) & 1);
+}
+
 // ---------------------------------------------------------------------------
 // Stream-K kernel.
 // ---------------------------------------------------------------------------
 template <typename T, int D, bool FUSED>
 __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
-    Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale,
-    int min_units, const T* new_k, const T* new_v) {
+    Dev d, int layer, const __grid_constant__ CUtensorMap map_lo,
+    const __grid_constant__ CUtensorMap map_hi, const T* __restrict__ q, T* __restrict__ out,
+    float qk_scale, int min_units, const T* new_k, const T* new_v) {
   using C = SkCfg<T, D>;
+  static_assert(!C::MMA, "the stream-K kernel runs the CUDA-core page loop");
   static_assert(C::WARPS == G, "the split-K merge maps one warp to one query row");
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -751,8 +1014,9 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
 // ---------------------------------------------------------------------------
 template <typename T, int D, bool FUSED, class C>
 __global__ void __launch_bounds__(C::THREADS) attn_decode_split_kernel(
-    Dev d, int layer, const T* __restrict__ q, T* __restrict__ out, float qk_scale, int k,
-    uint32_t epoch, const T* new_k, const T* new_v) {
+    Dev d, int layer, const __grid_constant__ CUtensorMap map_lo,
+    const __grid_constant__ CUtensorMap map_hi, const T* __restrict__ q, T* __restrict__ out,
+    float qk_scale, int k, uint32_t epoch, const T* new_k, const T* new_v) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const Smem<C> sm(smem, warp);
@@ -767,29 +1031,46 @@ __global__ void __launch_bounds__(C::THREADS) attn_decode_split_kernel(
   const int nb = si.n_blocks;
   const int b0 = (int)((int64_t)slice * nb / k), b1 = (int)((int64_t)(slice + 1) * nb / k);
   Segment<C> sg;
-  sg.init(d, si, head, b0, b1 - b0, warp);
+  sg.init(d, si, head, b0, b1 - b0, warp, &map_lo, &map_hi);
   sg.prefetch(d, layer, sm, 0, warp, lane);
   if (warp == 0) prefetch_q<C>(d, si, head, q, lane);
   pdl_wait();
-  float qr[G][2 * C::VEC];
-  load_q<C>(d, si, head, q, qk_scale, lane, qr);
-  float m_run = -INFINITY, l_run = 0.f;
-  float2 acc[G][C::PVD / 2];
+  int failed_at;
+  if constexpr (C::MMA) {
+    uint32_t qb[8][2];
+    load_q_mma<C>(d, si, head, q, qk_scale, lane, qb);
+    float m2[2] = {-INFINITY, -INFINITY}, l2[2] = {0.f, 0.f};
+    float o[8][4];
 #pragma unroll
-  for (int g = 0; g < G; ++g)
+    for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+    failed_at = stream_pages_mma<C, FUSED>(d, layer, sg, sm, 0, qb, m2, l2, o, warp, lane,
+                                           new_k, new_v);
+    if (failed_at >= 0) {
+      m2[0] = m2[1] = -INFINITY;
+      l2[0] = l2[1] = 0.f;
+    }
+    drain_after_failure<C>(d, sm, sg, failed_at);
+    __syncthreads();
+    publish_warp_mma<C>(sm, m2, l2, o, warp, lane);
+  } else {
+    float qr[G][2 * C::VEC];
+    load_q<C>(d, si, head, q, qk_scale, lane, qr);
+    float m_run = -INFINITY, l_run = 0.f;
+    float2 acc[G][C::PVD / 2];
 #pragma unroll
-    for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
-  const int failed_at = stream_pages<C, FUSED>(d, layer, sg, sm, 0, qr, m_run, l_run, acc, warp,
-                                               lane, new_k, new_v);
-  if (failed_at >= 0) {
-    // A wait gave up (error recorded): drain this warp's copies, contribute nothing.
-    for (int j = failed_at; j < min(sg.n_my, failed_at + C::STAGES); ++j)
-      mbar_wait(d, &sm.wbars[j % C::STAGES], (j / C::STAGES) & 1);
-    m_run = -INFINITY;
-    l_run = 0.f;
+    for (int g = 0; g < G; ++g)
+#pragma unroll
+      for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
+    failed_at = stream_pages<C, FUSED>(d, layer, sg, sm, 0, qr, m_run, l_run, acc, warp, lane,
+                                       new_k, new_v);
+    if (failed_at >= 0) {
+      m_run = -INFINITY;
+      l_run = 0.f;
+    }
+    drain_after_failure<C>(d, sm, sg, failed_at);
+    __syncthreads();
+    publish_warp<C>(sm, m_run, l_run, acc, warp, lane);
   }
-  __syncthreads();
-  publish_warp<C>(sm, m_run, l_run, acc, warp, lane);
   __syncthreads();
   merge_warps<C>(sm, warp, lane);
   T* orow = out + ((size_t)si.q_row0 * d.q_heads + head * G) * D;
@@ -867,7 +1148,7 @@ cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int
                           cudaStream_t s, uint32_t epoch, const void* new_k, const void* new_v) {
   static thread_local const int grid = stream_k_grid<T, D>(d);
   static thread_local const int slots = split_slots<T, D, SpCfg<T, D>>();
-  static thread_local const int slots4 = split_slots<T, D, SkCfg<T, D>>();
+  static thread_local const int slots4 = split_slots<T, D, Sp4Cfg<T, D>>();
   const float scale = LOG2E / sqrtf((float)D);
   const int n_pairs = n_seq * d.kv_heads;
   const T* qt = static_cast<const T*>(q);
@@ -875,25 +1156,33 @@ cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int
   const T* nk = static_cast<const T*>(new_k);
   const T* nv = static_cast<const T*>(new_v);
   const int k = n_pairs * SPLIT_MIN_K <= slots ? min(MAX_PARTS, slots / n_pairs) : 0;
+  const int k4 = k == 0 && n_pairs * SPLIT4_MIN_K <= slots4 ? min(MAX_PARTS, slots4 / n_pairs) : 0;
   const bool fused = nk != nullptr;
+  // Tensor maps of the pool for the tensor-core page loop (bfloat16).
+  CUtensorMap map_lo, map_hi;
+  memset(&map_lo, 0, sizeof(map_lo));
+  memset(&map_hi, 0, sizeof(map_hi));
+  if (((SpCfg<T, D>::MMA && k > 0) || (Sp4Cfg<T, D>::MMA && k4 > 0)) &&
+      !pool_tensor_maps(d, &map_lo, &map_hi))
+    return cudaErrorInvalidValue;
   if (k > 0) {
     using C = SpCfg<T, D>;
     return launch_ex(fused ? &attn_decode_split_kernel<T, D, true, C>
                            : &attn_decode_split_kernel<T, D, false, C>,
-                     dim3(n_pairs * k), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, qt, ot,
-                     scale, k, n_pairs * k <= d.dec_tag_slots ? epoch : 0u, nk, nv);
+                     dim3(n_pairs * k), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, map_lo,
+                     map_hi, qt, ot, scale, k, n_pairs * k <= d.dec_tag_slots ? epoch : 0u, nk,
+                     nv);
   }
-  const int k4 = n_pairs * SPLIT4_MIN_K <= slots4 ? min(MAX_PARTS, slots4 / n_pairs) : 0;
   if (k4 > 0) {
-    using C = SkCfg<T, D>;
+    using C = Sp4Cfg<T, D>;
     return launch_ex(fused ? &attn_decode_split_kernel<T, D, true, C>
                            : &attn_decode_split_kernel<T, D, false, C>,
-                     dim3(n_pairs * k4), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, qt, ot,
-                     scale, k4, 0u, nk, nv);
+                     dim3(n_pairs * k4), dim3(C::THREADS), C::SMEM, s, pdl, d, layer, map_lo,
+                     map_hi, qt, ot, scale, k4, 0u, nk, nv);
   }
   return launch_ex(fused ? &attn_decode_kernel<T, D, true> : &attn_decode_kernel<T, D, false>,
                    dim3(grid), dim3(SkCfg<T, D>::THREADS), SkCfg<T, D>::SMEM, s, pdl, d, layer,
-                   qt, ot, scale, DEC_MIN_UNITS, nk, nv);
+                   map_lo, map_hi, qt, ot, scale, DEC_MIN_UNITS, nk, nv);
 }
 
 }  // namespace

@@ -223,6 +223,20 @@ bool make_pool_maps(const Dev& d, PoolMaps& m) {
   return m.ok;
 }
 
+}  // namespace
+
+bool pool_tensor_maps(const Dev& d, CUtensorMap* lo, CUtensorMap* hi) {
+  static thread_local PoolMaps maps;
+  if (!maps.ok || maps.pool != d.pool) {
+    if (!make_pool_maps(d, maps)) return false;
+  }
+  *lo = maps.lo;
+  *hi = maps.hi;
+  return true;
+}
+
+namespace {
+
 template <int MT>
 int pf_grid(const void* fn, int threads, int smem) {
   cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -247,15 +261,13 @@ cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* ou
   (void)n_seq;
   (void)max_t;
   if (d.esz == 2) {
-    static thread_local PoolMaps maps;
     static thread_local int gtc = 0;
-    if (!maps.ok || maps.pool != d.pool) {
-      if (!make_pool_maps(d, maps)) return cudaErrorInvalidValue;
-    }
+    CUtensorMap lo, hi;
+    if (!pool_tensor_maps(d, &lo, &hi)) return cudaErrorInvalidValue;
     if (!gtc) gtc = pf_grid<0>(prefill_tc_kernel_ptr(), prefill_tc_threads(), prefill_tc_smem());
     // Each CTA of the stream-K split may write two partial slots.
-    return launch_attn_prefill_tc(d, layer, maps.lo, maps.hi, q, out,
-                                  std::min(gtc, d.max_pf_items / 2), pdl, s);
+    return launch_attn_prefill_tc(d, layer, lo, hi, q, out, std::min(gtc, d.max_pf_items / 2),
+                                  pdl, s);
   }
   const float scale = LOG2E / sqrtf((float)d.head_dim);
   static thread_local int gf = 0;

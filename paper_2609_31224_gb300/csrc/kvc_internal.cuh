@@ -353,6 +353,17 @@ __device__ inline void bulk_g2s(void* dst_smem, const void* src_gmem, uint32_t b
       : "memory");
 }
 
+// 2-D tensor copy (TMA engine) of the box at column x, row y of `map` into
+// shared memory, completing on `bar`.
+__device__ inline void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y,
+                                   uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
 // Programmatic dependent launch: let the next kernel in the stream start its
 // CTAs early, and wait until the previous kernel's writes are visible.
 __device__ inline void pdl_launch_dependents() {
@@ -455,6 +466,10 @@ cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& l
                                    const CUtensorMap& hi, const void* q, void* out, int grid,
                                    bool pdl, cudaStream_t s);
 const void* prefill_tc_kernel_ptr();
+// Two 2-D views of the bfloat16 pool as rows of 128 elements (columns 0-63 and
+// 64-127), 16-row boxes, 128-byte swizzle; cached per pool.  False if the driver
+// entry point is missing or the encoding fails.
+bool pool_tensor_maps(const Dev& d, CUtensorMap* lo, CUtensorMap* hi);
 int prefill_tc_smem();
 int prefill_tc_threads();
 int noalloc_max_pairs();
