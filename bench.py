@@ -37,13 +37,13 @@ UNIT = "audio-s/s"
 
 
 # DRAM bytes per algorithmic byte of the roofline kernel (reads + writes), from one
-# ncu capture of the 16-session, two-layer reduced case: 275.30 MB of traffic for a
-# 269.29 MB launch.  Valid only while the decode sources hash to the version it was
-# taken on; the roofline's traffic is null otherwise.
-DECODE_TRAFFIC_RATIO = 275.30 / 269.29
+# ncu capture of the stream-K kernel on the 24-session, two-layer reduced case:
+# 410.72 MB of traffic for a 403.97 MB launch.  Valid only while the decode sources
+# hash to the version it was taken on; the roofline's traffic is null otherwise.
+DECODE_TRAFFIC_RATIO = 410.72 / 403.97
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "ef88ea5f45197e0a7a0615a9ab72eea358e6cdb1da904905c924c575b0428cd0"
+DECODE_TRAFFIC_SHA256 = "76321e329058128d63dab61dfa347c95ad8981f30ca7d8ad21733a1a021824c8"
 
 
 def decode_traffic(alg_bytes_per_launch):

@@ -25,6 +25,9 @@
 
 #include "kvc_internal.cuh"
 
+// Shape constants of the CUDA-core loop are unused by the tensor-core shapes.
+#pragma nv_diag_suppress 177
+
 namespace kvc {
 
 namespace {
@@ -73,7 +76,8 @@ using SkCfg = DecCfg<T, D, 4, 2>;
 constexpr int SP_WARPS = 16, SP_STAGES = 1;
 template <typename T, int D>
 using SpCfg = DecCfg<T, D, SP_WARPS, SP_STAGES, true>;
-// Pair-split kernel for calls with too many pairs for SpCfg: stream-K's CTA shape.
+// Pair-split kernel for calls with too many pairs for SpCfg: stream-K's CTA shape,
+// with the CUDA-core page loop.
 constexpr bool SP4_MMA = false;
 template <typename T, int D>
 using Sp4Cfg = DecCfg<T, D, 4, 2, SP4_MMA>;
