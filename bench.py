@@ -162,6 +162,20 @@ def step_bytes(w, drv, st, prev_resident: dict) -> tuple[float, float, int]:
     return total, round0_bytes, round0_n
 
 
+def workload_config(w, start: int, steps: int, world: int, per_layer: bool) -> dict:
+    """The `config` object of the JSON line (both arms)."""
+    return {
+        "workload": w.name,
+        "sessions": w.n_sessions, "layers": w.layers, "q_heads": w.q_heads,
+        "kv_heads": w.kv_heads, "head_dim": w.head_dim, "page_size": w.page_size,
+        "budget": w.budget, "window": w.window, "units_per_session": w.units,
+        "offsets": f"U{{0..{w.offset_max}}}", "timed_steps": [start, start + steps],
+        "l2": "no flush: per-step K/V traffic >> 129 MB L2",
+        "parallelism": f"replicas x{world}",
+        "append": "per-layer" if per_layer else "whole chunk",
+    }
+
+
 def run_ours(args, rank: int, world: int, local_rank: int):
     import torch
     from synth import script as S
@@ -317,17 +331,8 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         "vs_baseline": None,
         "dtype": w.dtype,
         "data": "synthetic (seeded SplitMix64 Irwin-Hall values, PCG64 session scripts)",
-        "config": {
-            "workload": w.name,
-            "sessions": w.n_sessions, "layers": w.layers, "q_heads": w.q_heads,
-            "kv_heads": w.kv_heads, "head_dim": w.head_dim, "page_size": w.page_size,
-            "budget": w.budget, "window": w.window, "units_per_session": w.units,
-            "offsets": f"U{{0..{w.offset_max}}}", "timed_steps": [start, start + args.steps],
-            "audio_seconds_timed_per_gpu": audio_s,
-            "l2": "no flush: per-step K/V traffic >> 129 MB L2",
-            "parallelism": f"replicas x{world}",
-            "append": "per-layer" if args.per_layer_append else "whole chunk",
-        },
+        "config": dict(workload_config(w, start, args.steps, world, args.per_layer_append),
+                       audio_seconds_timed_per_gpu=audio_s),
         "path_hbm_gbs": (tot_bytes / 1e9) / (elapsed_ms / 1e3),
         "path_frac_of_peak": (tot_bytes / 1e9) / (elapsed_ms / 1e3) / peak,
         "roofline": {
@@ -582,21 +587,28 @@ def run_reference(args, rank: int, world: int):
     """The oracle timed as the reference arm (host cores), same metric and unit."""
     if rank != 0:
         return None
-    samples = [oracle_sample(layers_sampled=1, session=(i % 64)) for i in range(args.steps)]
-    for _ in range(0):
-        pass
+    from synth import script as S
+    w = S.BATCH64_BF16
+    start = S.steady_state_step(w, S.workload_scripts(w))
+    # Each step: one session-unit of the steady state, 1 of its 32 layers (sessions taken
+    # in turn); W untimed samples first.
+    for i in range(args.warmup):
+        oracle_sample(layers_sampled=1, session=(args.steps + i) % w.n_sessions)
+    samples = [oracle_sample(layers_sampled=1, session=i % w.n_sessions)
+               for i in range(args.steps)]
     total_audio = sum(s["value"] * s["seconds"] for s in samples)
     total_t = sum(s["seconds"] for s in samples)
     v = total_audio / total_t
+    sample = "1 of 32 layers of one session-unit per step (sessions in turn, step %d)" % start
     return {
         "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * total_t / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "impl": "reference",
-        "config": {"workload": "batch64-bf16-32L-32q8kv-d128-600u-off300-B4096-W10",
-                   "sample": "1 of 32 layers of one session-unit per step"},
+        "data": "synthetic (seeded SplitMix64 Irwin-Hall values, PCG64 session scripts)",
+        "impl": "reference",
+        "config": dict(workload_config(w, start, args.steps, world, False), sample=sample),
         "cpu_baseline": {"value": v, "unit": UNIT, "kind": "oracle",
-                         "cores": samples[0]["cores"], "sample": samples[0]["sample"]},
+                         "cores": samples[0]["cores"], "sample": sample},
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
