@@ -203,9 +203,14 @@ int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out
 /* Single-token decode GQA attention of one layer (transcript, delimiter and
  * response tokens): the last append gave each of its n_seq sessions exactly
  * one token; that token attends to every resident key, itself included.
- * Split-K over pages with a log-sum-exp merge.
+ * Split-K over pages with a log-sum-exp merge; for bfloat16 calls of at most
+ * 9 sessions the page products run on tensor cores (q and P rounded to
+ * bfloat16, binary32 accumulation).
  *   d_q     device [n_seq][Hq][D] un-rotated queries (call order of the append)
- *   d_out   device [n_seq][Hq][D] */
+ *   d_out   device [n_seq][Hq][D]
+ * May be captured into a CUDA graph: a launch made while `stream` is capturing
+ * merges its split-K parts with an acquire-release arrival, so replays are
+ * correct; eager launches tag their parts with a per-context launch counter. */
 int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void* stream);
 
 /* kvc_attn_decode without caller-provided scratch.  The paper has no
