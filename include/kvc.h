@@ -29,6 +29,11 @@
  *    reports the recorded code).
  *  - Layouts are row-major and contiguous.  The element type (binary32 or
  *    bfloat16) is fixed at creation for K, V, q and out alike.
+ *  - One context serves one host thread and one stream at a time: its
+ *    launches share the context's scratch (split-K slots, arrival counters)
+ *    and its host mirrors, so calls on it must be ordered on one stream (or
+ *    on streams ordered by events) and not made concurrently.  Independent
+ *    contexts share nothing.
  */
 #ifndef KVC_H
 #define KVC_H
