@@ -162,6 +162,22 @@ def step_bytes(w, drv, st, prev_resident: dict) -> tuple[float, float, int]:
     return total, round0_bytes, round0_n
 
 
+def job_throughput(units: float, elapsed_ms: float, world: int) -> tuple[float, float]:
+    """Whole-job throughput: the units all ranks processed over the slowest rank's time.
+    Returns (units per second, max elapsed ms).  With world > 1 it reduces over the
+    default process group (NCCL: CUDA tensors, gloo: host tensors)."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+        u = torch.tensor([float(units)], dtype=torch.float64, device=dev)
+        t = torch.tensor([float(elapsed_ms)], dtype=torch.float64, device=dev)
+        dist.all_reduce(u, op=dist.ReduceOp.SUM)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        units, elapsed_ms = float(u.item()), float(t.item())
+    return units / (elapsed_ms / 1e3), elapsed_ms
+
+
 def workload_config(w, start: int, steps: int, world: int, per_layer: bool) -> dict:
     """The `config` object of the JSON line (both arms)."""
     return {
@@ -279,13 +295,8 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     if world > 1:
         torch.distributed.barrier()
     clk = clocks.stop()
-    elapsed_ms = t0.elapsed_time(t1)
-    if world > 1:
-        tt = torch.tensor([elapsed_ms], dtype=torch.float64, device="cuda")
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        elapsed_ms = float(tt.item())
     audio_s = sum(len(st.pairs) for st in timed)          # one unit = one audio second
-    value_rank = audio_s / (elapsed_ms / 1e3)
+    value, elapsed_ms = job_throughput(audio_s, t0.elapsed_time(t1), world)
 
     # Algorithmic bytes (attention reads every resident K/V byte once per call per layer).
     res = n_res_buf.cpu().numpy()
@@ -320,7 +331,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     dec_gbs = (sum(dec_bytes) / 1e9) / (sum(dec_times) / 1e3) if dec_times else None
     out = {
         "metric": METRIC,
-        "value": value_rank * world,
+        "value": value,
         "unit": UNIT,
         "n_gpus": world,
         "steps": args.steps,
@@ -429,12 +440,9 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
     wall = time.perf_counter() - t0
     copy_ms = [a.elapsed_time(b) for a, b in zip(copy_start, ready)]
     comp_ms = [a.elapsed_time(b) for a, b in comp]
-    if world > 1:
-        tt = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
     audio_s = sum(len(st.pairs) for st in steps)
-    return {"value": world * audio_s / (ms / 1e3), "unit": UNIT,
+    value, ms = job_throughput(audio_s, ms, world)
+    return {"value": value, "unit": UNIT,
             "h2d_bytes_per_step": h2d_total / n_steps, "d2h_bytes_per_step": d2h_total / n_steps,
             "steps": n_steps, "first_step": first_step, "host_wall_s": wall,
             "host_submit_ms_per_step": 1e3 * submit / n_steps,
