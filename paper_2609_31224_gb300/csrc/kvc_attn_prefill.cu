@@ -200,14 +200,19 @@ EncodeTiledFn get_encode() {
 
 struct PoolMaps {
   const uint8_t* pool = nullptr;
+  uint64_t rows = 0;
   CUtensorMap lo, hi;
   bool ok = false;
 };
 
+uint64_t pool_rows(const Dev& d) {
+  return (uint64_t)d.n_pages * d.layers * 2 * d.kv_heads * PS;
+}
+
 bool make_pool_maps(const Dev& d, PoolMaps& m) {
   EncodeTiledFn enc = get_encode();
   if (!enc) return false;
-  const uint64_t rows = (uint64_t)d.n_pages * d.layers * 2 * d.kv_heads * PS;
+  const uint64_t rows = pool_rows(d);
   cuuint64_t dims[2] = {64, rows};
   cuuint64_t strides[1] = {(cuuint64_t)PF_D * 2};
   cuuint32_t box[2] = {64, PS};
@@ -220,14 +225,17 @@ bool make_pool_maps(const Dev& d, PoolMaps& m) {
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   m.ok = (r1 == CUDA_SUCCESS && r2 == CUDA_SUCCESS);
   m.pool = d.pool;
+  m.rows = rows;
   return m.ok;
 }
 
 }  // namespace
 
 bool pool_tensor_maps(const Dev& d, CUtensorMap* lo, CUtensorMap* hi) {
+  // Keyed on the pool's address and extent: a later context may get the same address
+  // for a pool of another shape.
   static thread_local PoolMaps maps;
-  if (!maps.ok || maps.pool != d.pool) {
+  if (!maps.ok || maps.pool != d.pool || maps.rows != pool_rows(d)) {
     if (!make_pool_maps(d, maps)) return false;
   }
   *lo = maps.lo;
