@@ -83,7 +83,8 @@ class OracleCache:
         for s in sessions:
             for pid in self.layout[s].hist_pages + self.layout[s].live_pages:
                 self.pool.release(pid)
-            self.policy[s] = SessionPolicy(self.cfg.budget, self.cfg.window)
+            self.policy[s] = SessionPolicy(self.cfg.budget, self.cfg.window, self.cfg.policy,
+                                           self.cfg.sink, self.cfg.recent)
             self.layout[s] = SessionLayout(self.cfg.page_size)
         self.last_append = None
 
@@ -110,6 +111,7 @@ class OracleCache:
             "live_pages": list(lay.live_pages),
             "resident": pol.resident(),
             "n_evicted": pol.pos_next - pol.resident(),
+            "peak_resident": pol.peak_resident,
             "pos": pos,
             "type": [pol.type[p] for p in pos],
             "unit": [pol.unit[p] for p in pos],

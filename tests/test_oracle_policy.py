@@ -432,3 +432,78 @@ def test_transcript_export_keeps_every_transcript(policy):
     for s in (0, 1):
         assert c.transcript_positions(s) == fed[s]
         assert any(c.policy[s].evicted)
+
+
+# -- release -------------------------------------------------------------------------------
+
+def _unit_chunk(rng, text=False):
+    unit = [ACOUSTIC | UNIT_BEGIN] + [ACOUSTIC] * int(rng.integers(0, 9)) + [ASR_DELIM] + \
+        [TRANSCRIPT] * int(rng.poisson(2)) + [ASR_DELIM]
+    return unit + ([TEXT] * int(rng.integers(1, 6)) if text else [])
+
+
+@pytest.mark.parametrize("policy,sink,recent", [("unit", 0, 0), ("position", 0, 0),
+                                                ("sink_recent", 3, 25)])
+def test_release_then_refeed_equals_a_fresh_session(policy, sink, recent):
+    """A released session starts over under the cache's own policy: fed the same units
+    afterwards it evicts exactly what a fresh session fed those units evicts (policy
+    record, peak, frontier), its page lists have the same shape, and every page it held
+    went back to the pool.  A release that rebuilt the session under the default rule
+    would diverge from the fresh position-granular or sink + recent session at its first
+    evict past the budget."""
+    budget, window, ps = 20, 1, 4
+
+    def cache(n_sessions):
+        return OracleCache(OracleConfig(n_sessions=n_sessions, layers=1, q_heads=1, kv_heads=1,
+                                        head_dim=4, page_size=ps, budget=budget, window=window,
+                                        dtype="f32", rope_base=10000.0, n_pages=400,
+                                        policy=policy, sink=sink, recent=recent))
+
+    rng = np.random.default_rng(5)
+    before = [_unit_chunk(rng, text=(i % 7 == 3)) for i in range(25)]
+    after = [_unit_chunk(rng, text=(i % 5 == 2)) for i in range(30)]
+    other = [_unit_chunk(rng) for _ in range(25)]
+    used = cache(2)
+    for a, b in zip(before, other):
+        used.append_chunk([0, 1], [a, b])
+        used.evict([0, 1])
+    assert any(used.policy[0].evicted)
+    free_before = used.pool.free_count()
+    held = len(used.layout[0].hist_pages) + len(used.layout[0].live_pages)
+    used.release([0])
+    assert used.pool.free_count() == free_before + held
+    assert used.state(0)["pos_next"] == 0 and used.state(0)["peak_resident"] == 0
+    fresh = cache(1)
+    for a in after:
+        used.append_chunk([0], [a])
+        fresh.append_chunk([0], [a])
+        assert used.evict([0]) == fresh.evict([0])
+        pu, pf = used.policy[0], fresh.policy[0]
+        assert (pu.policy, pu.sink, pu.recent) == (policy, sink, recent)
+        assert pu.evicted == pf.evicted and pu.frontier == pf.frontier
+        su, sf = used.state(0), fresh.state(0)
+        for key in ("pos_next", "unit_cur", "n_hist", "live_head", "n_live", "resident",
+                    "n_evicted", "peak_resident", "pos", "type", "unit"):
+            assert su[key] == sf[key], key
+        assert len(su["hist_pages"]) == len(sf["hist_pages"])
+        assert len(su["live_pages"]) == len(sf["live_pages"])
+    assert any(fresh.policy[0].evicted)
+
+
+def test_release_of_the_only_session_restores_the_page_ids():
+    """With one session, a release frees the whole pool, so the lowest-free-id allocator
+    hands out the same page ids as in a fresh cache."""
+    rng = np.random.default_rng(9)
+    units = [_unit_chunk(rng, text=(i % 6 == 0)) for i in range(20)]
+    a, b = _cache(15, 2), _cache(15, 2)
+    for u in units[:12]:
+        a.append_chunk([0], [u])
+        a.evict([0])
+    a.release([0])
+    assert a.pool.free_count() == a.pool.n_pages
+    for u in units:
+        a.append_chunk([0], [u])
+        b.append_chunk([0], [u])
+        a.evict([0])
+        b.evict([0])
+        assert a.state(0) == b.state(0)
