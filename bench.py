@@ -38,12 +38,12 @@ UNIT = "audio-s/s"
 
 # DRAM bytes per algorithmic byte of the roofline kernel (reads + writes), from one
 # ncu capture of the stream-K kernel on the 24-session, two-layer reduced case:
-# 410.72 MB of traffic for a 403.97 MB launch.  Valid only while the decode sources
+# 410.93 MB of traffic (406.82 MB read, 4.11 MB written) for a 403.97 MB launch.  Valid only while the decode sources
 # hash to the version it was taken on; the roofline's traffic is null otherwise.
-DECODE_TRAFFIC_RATIO = 410.72 / 403.97
+DECODE_TRAFFIC_RATIO = 410.93 / 403.97
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "76321e329058128d63dab61dfa347c95ad8981f30ca7d8ad21733a1a021824c8"
+DECODE_TRAFFIC_SHA256 = "f36ab38985938043022c24377366d8409783aba1dc77a03b1f3530905e77c25c"
 
 
 def decode_traffic(alg_bytes_per_launch):
@@ -461,6 +461,8 @@ def run_unbounded_comparison() -> dict:
     from synth import script as S
     from synth.driver import Driver
     res = {}
+    clocks = Clocks(torch.cuda.current_device())
+    clocks.start()
     for w in (S.SINGLE_BF16, S.SINGLE_BF16_UNBOUNDED):
         scripts = S.workload_scripts(w)
         drv = Driver(w, scripts)
@@ -488,8 +490,10 @@ def run_unbounded_comparison() -> dict:
         }
         del drv
         torch.cuda.empty_cache()
+    clk = clocks.stop()
     b, f = res[S.SINGLE_BF16.name], res[S.SINGLE_BF16_UNBOUNDED.name]
     return {"comparison": "single session, B=4096 vs B=infinity, same seeded inputs",
+            "clocks": clk,
             "units": S.SINGLE_BF16.units, "runs": res,
             "peak_kv_reduction": 1.0 - b["peak_kv_bytes"] / f["peak_kv_bytes"],
             "attention_time_ratio_full_over_budget": f["attention_ms"] / b["attention_ms"]}
@@ -499,13 +503,16 @@ def run_unbounded_comparison() -> dict:
 def run_budget_sweep(n_sessions: int) -> dict:
     """Budgets B in {unbounded, 8K, 6K, 4K, 0 (floor)} on full-size single sessions (32
     layers, 600 units, batch size 1, one session at a time): End and Peak resident
-    positions (means over sessions) and the path's GPU time per unit (append, every
-    layer's attention and the evict of one unit; CUDA events), mean and p99."""
+    positions (means over sessions, as the device reports them) and the path's GPU time per
+    unit (append, every layer's attention and the evict of one unit; CUDA events), mean and
+    p99.  SM clocks are sampled throughout."""
     import numpy as np
     import torch
     from synth import script as S
     from synth.driver import Driver
     rows = []
+    clocks = Clocks(torch.cuda.current_device())
+    clocks.start()
     for budget in (-1, 8192, 6144, 4096, 0):
         w = S.SINGLE_BF16.with_(name=f"single-bf16-32L-600u-B{budget}-W10", budget=budget,
                                 n_sessions=n_sessions)
@@ -532,26 +539,33 @@ def run_budget_sweep(n_sessions: int) -> dict:
         t = np.array(unit_ms)
         rows.append({"budget": "unbounded" if budget < 0 else budget,
                      "end_positions": float(np.mean(ends)), "peak_positions": float(np.mean(peaks)),
+                     "end_per_session": ends, "peak_per_session": peaks,
                      "unit_ms_mean": float(t.mean()), "unit_ms_p99": float(np.percentile(t, 99)),
                      "units": int(t.size)})
+    clk = clocks.stop()
+    full = rows[0]["peak_positions"]
+    for r in rows:
+        r["peak_reduction_vs_unbounded"] = 1.0 - r["peak_positions"] / full
     return {"sweep": "Table-3-shaped budget sweep, synthetic single-session workload "
                      "(32 layers, 32/8 heads, D=128, bf16, W=10, 600 units, batch size 1)",
-            "sessions_per_budget": n_sessions, "rows": rows}
+            "data": "synthetic (seeded SplitMix64 Irwin-Hall values, PCG64 session scripts)",
+            "sessions_per_budget": n_sessions, "rows": rows, "clocks": clk}
 
 
 # -- the oracle on the host cores -----------------------------------------------------------------
-def oracle_sample(layers_sampled: int = 1, session: int = 0, start: int | None = None) -> dict:
-    """Time the CPU oracle on one session's unit at the benchmark's steady state, for
-    `layers_sampled` of its 32 layers (policy + every attention call of those layers);
-    scaled to audio-s/s by the sampled fraction of one unit."""
+_BLAS_THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
+
+
+def _oracle_layers(session: int, start: int, layers: list) -> float:
+    """One session's unit at step `start` of the 64-session workload through the oracle:
+    the state before the unit is built untimed, then the unit's policy steps and every
+    attention call of `layers` are timed.  Returns the timed seconds."""
     from oracle.cache import OracleCache, OracleConfig
     from synth import script as S
     from synth import values as V
 
     w = S.BATCH64_BF16
-    scripts = S.workload_scripts(w)
-    sc = scripts[session]
-    start = S.steady_state_step(w, scripts) if start is None else start
+    sc = S.session_script(w, session)
     unit = start - sc.offset
     orc = OracleCache(OracleConfig(n_sessions=1, layers=w.layers, q_heads=w.q_heads,
                                    kv_heads=w.kv_heads, head_dim=w.head_dim,
@@ -572,23 +586,65 @@ def oracle_sample(layers_sampled: int = 1, session: int = 0, start: int | None =
     for types in chunks:
         orc.append_chunk([0], [types])
         pos = orc.last_append[0][1]
-        for layer in range(layers_sampled):
+        for layer in layers:
             q = V.layer_tensor(w.seed, V.TAG_Q, session, layer, pos, w.q_heads, w.head_dim,
                                w.dtype)
             orc.attend(layer, [q], kv)
     orc.evict([0])
-    dt = time.perf_counter() - t0
-    frac = layers_sampled / w.layers
+    return time.perf_counter() - t0
+
+
+def oracle_sample(layers_sampled: int = 1, session: int = 0, start: int | None = None,
+                  workers: int = 1) -> dict:
+    """Time the CPU oracle on one session's unit at the benchmark's steady state, for
+    `layers_sampled` of its 32 layers (policy + every attention call of those layers),
+    scaled to audio-s/s by the sampled fraction of one unit.
+
+    workers = 1: one process with single-threaded BLAS.  workers = N: N processes
+    (spawned; each single-threaded), layer i in process i % N, all replaying the unit's
+    calls in parallel; the value is the sampled fraction over the wall time of the
+    parallel part."""
+    import multiprocessing as mp
+    from synth import script as S
+    w = S.BATCH64_BF16
+    if start is None:
+        start = S.steady_state_step(w, S.workload_scripts(w))
+    unit = start - S.session_script(w, session).offset
+    n_calls = 1 + len(S.session_script(w, session).decode_types(unit))
+    saved = {k: os.environ.get(k) for k in _BLAS_THREAD_VARS}
+    for k in _BLAS_THREAD_VARS:
+        os.environ[k] = "1"
     try:
-        from threadpoolctl import threadpool_info
-        cores = max([i.get("num_threads", 1) for i in threadpool_info()] + [1])
-    except Exception:
-        cores = len(os.sched_getaffinity(0))
-    return {"value": frac / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(workers) as pool:
+            pool.apply(time.perf_counter)        # workers started before the clock
+            parts = [list(range(i, layers_sampled, workers)) for i in range(workers)]
+            t0 = time.perf_counter()
+            pool.starmap(_oracle_layers, [(session, start, p) for p in parts if p])
+            dt = time.perf_counter() - t0
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    frac = layers_sampled / w.layers
+    return {"value": frac / dt, "unit": UNIT, "cores": workers, "kind": "oracle",
             "seconds": dt,
             "sample": f"session {session}, unit {unit} (step {start}) of {w.name}: eviction rule "
-                      f"+ {len(chunks)} attention calls x {layers_sampled}/{w.layers} layers "
-                      f"in float64; value = sampled fraction of one audio-second / time"}
+                      f"+ {n_calls} attention calls x {layers_sampled}/{w.layers} layers in "
+                      f"float64, {workers} single-threaded process(es); value = sampled "
+                      f"fraction of one audio-second / wall time"}
+
+
+def cpu_baseline() -> dict:
+    """The oracle on all host cores (the reported figure) and on one core."""
+    cores = len(os.sched_getaffinity(0))
+    allc = oracle_sample(layers_sampled=2 * cores, workers=cores)
+    one = oracle_sample(layers_sampled=6, workers=1)
+    allc["single_thread"] = {"value": one["value"], "cores": 1, "seconds": one["seconds"],
+                             "sample": one["sample"]}
+    return allc
 
 
 def run_reference(args, rank: int, world: int):
@@ -600,14 +656,17 @@ def run_reference(args, rank: int, world: int):
     start = S.steady_state_step(w, S.workload_scripts(w))
     # Each step: one session-unit of the steady state, 1 of its 32 layers (sessions taken
     # in turn); W untimed samples first.
+    cores = len(os.sched_getaffinity(0))
     for i in range(args.warmup):
-        oracle_sample(layers_sampled=1, session=(args.steps + i) % w.n_sessions)
-    samples = [oracle_sample(layers_sampled=1, session=i % w.n_sessions)
-               for i in range(args.steps)]
+        oracle_sample(layers_sampled=cores, session=(args.steps + i) % w.n_sessions,
+                      start=start, workers=cores)
+    samples = [oracle_sample(layers_sampled=cores, session=i % w.n_sessions, start=start,
+                             workers=cores) for i in range(args.steps)]
     total_audio = sum(s["value"] * s["seconds"] for s in samples)
     total_t = sum(s["seconds"] for s in samples)
     v = total_audio / total_t
-    sample = "1 of 32 layers of one session-unit per step (sessions in turn, step %d)" % start
+    sample = ("%d of 32 layers of one session-unit per step (sessions in turn, step %d), one "
+              "layer per single-threaded process on %d host cores" % (cores, start, cores))
     return {
         "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * total_t / args.steps,
@@ -672,7 +731,7 @@ def main():
     out = run_ours(args, rank, world, local_rank)
     if rank == 0:
         if world == 1 and not args.no_cpu_baseline:
-            out["cpu_baseline"] = oracle_sample(layers_sampled=20)
+            out["cpu_baseline"] = cpu_baseline()
         print(json.dumps(out))
     if world > 1:
         import torch

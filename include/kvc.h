@@ -193,10 +193,17 @@ int kvc_evict(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, int64_t* d_res
               void* stream);
 
 /* Chunked-prefill GQA attention of one layer for the queries of the last
- * appended chunk (e.g. the 17 acoustic positions of a unit): query t of a
- * session sits at its position and sees every resident key at or before it
- * (causal inside the chunk).  softmax(RoPE(q) . k / sqrt(D)) v, softmax in
- * binary32, K/V products on tensor cores for bfloat16.
+ * appended chunk.  Sec. 3.1: the model consumes speech in one-second duplex units
+ * (a unit marker, about ten audio tokens and the native decision, 17 positions in
+ * the workloads here), so each unit's positions enter the language model together
+ * as one chunk.  Sec. 3.3: attention runs over whatever the online eviction left
+ * resident, and the kept keys are used at their original rotary positions, never
+ * re-encoded.  Query t of a session sits at its own position and sees every
+ * resident key at or before it (causal inside the chunk):
+ * softmax(RoPE(q, p_t) . k / sqrt(D)) v, with the keys stored already rotated at
+ * their positions.  Softmax in binary32; for bfloat16 the q.k and P.v products run
+ * on tensor cores (tcgen05) with q and P rounded to bfloat16 and binary32
+ * accumulation; binary32 calls stay on CUDA cores.
  *   layer   0 .. L-1
  *   d_q     device [total][Hq][D] un-rotated queries, total and order as in
  *           the last kvc_append_chunk; chunks of at most 32 tokens
@@ -205,12 +212,21 @@ int kvc_evict(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, int64_t* d_res
 int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out,
                            void* stream);
 
-/* Single-token decode GQA attention of one layer (transcript, delimiter and
- * response tokens): the last append gave each of its n_seq sessions exactly
- * one token; that token attends to every resident key, itself included.
- * Split-K over pages with a log-sum-exp merge; for bfloat16 calls of at most
- * 9 sessions the page products run on tensor cores (q and P rounded to
- * bfloat16, binary32 accumulation).
+/* Single-token decode GQA attention of one layer.  Sec. 3.1: after the unit's
+ * first decision the model decodes, one token at a time, the transcription
+ * segment (<|asr_start|>, up to 64 transcript tokens, <|asr_end|>) and, in SPEAK
+ * units, the response text.  Sec. 3.3: each such token attends to the retained
+ * cache (the system prefix, transcripts and text of every unit, and the acoustic
+ * states of the units the eviction has not reached) with the kept keys at their
+ * original rotary positions.  The last append gave each of its n_seq sessions
+ * exactly one token; that token attends to every resident key, itself included.
+ * Split-K over pages with a log-sum-exp merge.
+ * Precision depends on the call's size: for bfloat16 calls of at most 9 sessions
+ * (8 KV heads, 152 SMs: while every (session, KV head) pair gets two one-CTA-per-SM
+ * slices) the page products run on tensor cores with q and P rounded to bfloat16
+ * and binary32 accumulation; larger calls keep q and P in binary32 on CUDA cores.
+ * So the same session's output can differ in the last bits with the number of
+ * sessions sharing its call; both stay within the attention tolerance.
  *   d_q     device [n_seq][Hq][D] un-rotated queries (call order of the append)
  *   d_out   device [n_seq][Hq][D]
  * May be captured into a CUDA graph: a launch made while `stream` is capturing
@@ -228,16 +244,19 @@ int kvc_attn_decode(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void*
  * Same arguments, layouts and result as kvc_attn_decode (within the attention
  * tolerance: the split-K chunking differs).  The split-K partial results and
  * arrival counters live in one fixed array in device global memory that the
- * library defines (8.1 MiB; every GPU that loads the library holds it until the
- * process exits), so this call allocates nothing.
+ * library defines (8.1 MiB in each CUDA context that loads the library, held until
+ * the context is destroyed or the process exits), so this call allocates nothing.
  *   - Limit: at most 4096 (session, kv-head) pairs per call, i.e. the last
  *     append's n_seq * kv_heads <= 4096; larger calls return KVC_EINVAL with a
  *     message and launch nothing.
- *   - The first call on each device looks up the array's device address (with
- *     that device current); make that first call before any stream capture.
- *   - Every call shares the array and clears the counters it needs; calls whose
- *     kernels can overlap on the GPU (other streams, other contexts in this
- *     process) race on it, so serialise them. */
+ *   - Each CUDA context holds its own copy of the array (runtime-API callers share
+ *     one primary context per device).  The first call made in a context, with
+ *     that context current, looks up the array's device address there (and the
+ *     SM count and the kernel's occupancy); make that first call before any
+ *     stream capture.
+ *   - Every call shares its context's array and clears the counters it needs;
+ *     calls whose kernels can overlap on the GPU (other streams, other library
+ *     contexts over the same CUDA context) race on it, so serialise them. */
 int kvc_attn_decode_noalloc(kvc_ctx* ctx, int layer, const void* d_q, void* d_out, void* stream);
 
 /* Resident count of one session (n_hist + n_live), including the system

@@ -503,8 +503,7 @@ int kvc_attn_decode_noalloc(kvc_ctx* ctx, int layer, const void* d_q, void* d_ou
                 "kvc_attn_decode_noalloc handles at most %d (session, kv-head) pairs per call; "
                 "this call has %d sessions x %d kv heads = %d",
                 noalloc_max_pairs(), ctx->last_n_seq, ctx->cfg.kv_heads, pairs);
-  const int cs = noalloc_chunks(ctx->d, ctx->last_n_seq);
-  KVC_CUDA(launch_attn_decode_noalloc(ctx->d, layer, d_q, d_out, ctx->last_n_seq, cs,
+  KVC_CUDA(launch_attn_decode_noalloc(ctx->d, layer, d_q, d_out, ctx->last_n_seq,
                                       static_cast<cudaStream_t>(stream)));
   return KVC_OK;
 }

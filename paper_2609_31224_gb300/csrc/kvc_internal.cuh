@@ -473,9 +473,8 @@ bool pool_tensor_maps(const Dev& d, CUtensorMap* lo, CUtensorMap* hi);
 int prefill_tc_smem();
 int prefill_tc_threads();
 int noalloc_max_pairs();
-int noalloc_chunks(const Dev& d, int n_seq);
 cudaError_t launch_attn_decode_noalloc(const Dev& d, int layer, const void* q, void* out,
-                                       int n_seq, int cs, cudaStream_t s);
+                                       int n_seq, cudaStream_t s);
 int prefill_grid_ctas(const Dev& d);
 
 }  // namespace kvc

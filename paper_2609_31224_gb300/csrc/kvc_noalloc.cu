@@ -4,11 +4,13 @@
 // global memory owned by this library, instead of in the caller's metadata
 // workspace.  The entry point allocates nothing.
 //
-// The array is a file-scope static __device__ object: every GPU that loads the
-// library holds it (NOALLOC_SCRATCH_BYTES) until the process exits.  All calls
-// share it, so calls whose kernels overlap on the GPU (different streams, or
-// different contexts of the same process) race on it and must be serialised by
-// the caller.
+// The array is a file-scope static __device__ object: every CUDA context that
+// loads the library (one per device for runtime-API callers, who share the
+// device's primary context) holds its own copy (NOALLOC_SCRATCH_BYTES) until the
+// context is destroyed or the process exits.  All calls in one context share that
+// copy, so calls whose kernels overlap on the GPU (different streams, or
+// different library contexts over the same CUDA context) race on it and must be
+// serialised by the caller.
 #include <algorithm>
 #include <mutex>
 
@@ -347,48 +349,112 @@ __global__ void __launch_bounds__(NA_THREADS) attn_decode_noalloc_kernel(
   }
 }
 
-// Device address of the static scratch, looked up once per device (with that
-// device current) on the first call made on it.
-constexpr int NA_MAX_DEVICES = 64;
-void* g_scratch_ptr[NA_MAX_DEVICES] = {};
-std::mutex g_scratch_mu;
+// Per-CUDA-context set-up, done by the first call made in a context (with that
+// context current): the array's device address in this context (each context
+// loads its own copy of the module), the SM count, and, for each kernel instance,
+// the shared-memory attribute and its resident CTAs per SM.  Contexts are told
+// apart by their unique id (cuCtxGetId), which is never reused, so a context that
+// replaces a destroyed one at the same address gets its own set-up.
+struct NaSetup {
+  unsigned long long ctx_id;
+  uint8_t* scratch;
+  int sms;
+  int per_sm[2];  // [0] binary32 / D = 64, [1] bfloat16 / D = 128
+};
+constexpr int NA_MAX_CONTEXTS = 64;
+NaSetup g_setup[NA_MAX_CONTEXTS];
+int g_n_setup = 0;
+std::mutex g_setup_mu;
 
-cudaError_t scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+typedef CUresult (*PfnCtxGetCurrent)(CUcontext*);
+typedef CUresult (*PfnCtxGetId)(CUcontext, unsigned long long*);
+
+cudaError_t driver_fn(const char* name, void** fn) {
+  cudaDriverEntryPointQueryResult q;
+  cudaError_t e = cudaGetDriverEntryPoint(name, fn, cudaEnableDefault, &q);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= NA_MAX_DEVICES) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_ptr[dev] = p;
-  }
-  *out = g_scratch_ptr[dev];
-  return cudaSuccess;
+  return (q == cudaDriverEntryPointSuccess && *fn) ? cudaSuccess : cudaErrorNotSupported;
 }
 
 template <typename T, int D>
-cudaError_t launch_typed(const Dev& d, int layer, const void* q, void* out, int n_seq, int cs,
-                         uint8_t* scratch, cudaStream_t s) {
+cudaError_t kernel_per_sm(int* per_sm) {
   const void* fn = reinterpret_cast<const void*>(&attn_decode_noalloc_kernel<T, D>);
   const int smem = NaCfg<T, D>::SMEM;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  int per_sm = 0, dev = 0, sms = 0;
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, NA_THREADS, smem);
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int grid = std::max(1, per_sm) * sms;
-  float* part_o = reinterpret_cast<float*>(scratch);
-  float2* part_ml = reinterpret_cast<float2*>(scratch + NA_PART_O_BYTES);
-  int32_t* count = reinterpret_cast<int32_t*>(scratch + NA_PART_O_BYTES + NA_PART_ML_BYTES);
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(per_sm, fn, NA_THREADS, smem);
+  if (e != cudaSuccess) return e;
+  return *per_sm > 0 ? cudaSuccess : cudaErrorInvalidConfiguration;
+}
+
+cudaError_t setup_for_current_context(NaSetup* out) {
+  static PfnCtxGetCurrent get_current = nullptr;
+  static PfnCtxGetId get_id = nullptr;
+  std::lock_guard<std::mutex> lock(g_setup_mu);
+  cudaError_t e;
+  if (!get_current || !get_id) {
+    void* f1 = nullptr;
+    void* f2 = nullptr;
+    if ((e = driver_fn("cuCtxGetCurrent", &f1)) != cudaSuccess) return e;
+    if ((e = driver_fn("cuCtxGetId", &f2)) != cudaSuccess) return e;
+    get_current = reinterpret_cast<PfnCtxGetCurrent>(f1);
+    get_id = reinterpret_cast<PfnCtxGetId>(f2);
+  }
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  void* p = nullptr;
+  if (!ctx) {
+    // No context current on this thread yet: the runtime makes the device's
+    // primary context current on this lookup.
+    if ((e = cudaGetSymbolAddress(&p, g_noalloc_scratch)) != cudaSuccess) return e;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx) return cudaErrorDeviceUninitialized;
+  }
+  unsigned long long id = 0;
+  if (get_id(ctx, &id) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  for (int i = 0; i < g_n_setup; ++i)
+    if (g_setup[i].ctx_id == id) {
+      *out = g_setup[i];
+      return cudaSuccess;
+    }
+  NaSetup s = {};
+  s.ctx_id = id;
+  if ((e = cudaGetSymbolAddress(&p, g_noalloc_scratch)) != cudaSuccess) return e;
+  s.scratch = static_cast<uint8_t*>(p);
+  int dev = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&s.sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+    return e;
+  if ((e = kernel_per_sm<float, 64>(&s.per_sm[0])) != cudaSuccess) return e;
+  if ((e = kernel_per_sm<__nv_bfloat16, 128>(&s.per_sm[1])) != cudaSuccess) return e;
+  // A full table only means later contexts repeat the set-up on every call.
+  if (g_n_setup < NA_MAX_CONTEXTS) g_setup[g_n_setup++] = s;
+  *out = s;
+  return cudaSuccess;
+}
+
+// Chunks per session: about four work items per resident CTA over the call,
+// limited by the static scratch and by NA_MAX_CHUNKS.
+int noalloc_chunks(int pairs, int resident_ctas) {
+  int cs = std::max(1, 4 * resident_ctas / std::max(1, pairs));
+  cs = std::min(cs, NA_MAX_CHUNKS);
+  cs = std::min(cs, NA_MAX_SLOTS / std::max(1, pairs));
+  return std::max(1, cs);
+}
+
+template <typename T, int D>
+cudaError_t launch_typed(const Dev& d, int layer, const void* q, void* out, int n_seq,
+                         const NaSetup& su, cudaStream_t s) {
+  const int per_sm = su.per_sm[sizeof(T) == 2 ? 1 : 0];
+  const int grid = per_sm * su.sms;
+  const int cs = noalloc_chunks(n_seq * d.kv_heads, grid);
+  float* part_o = reinterpret_cast<float*>(su.scratch);
+  float2* part_ml = reinterpret_cast<float2*>(su.scratch + NA_PART_O_BYTES);
+  int32_t* count = reinterpret_cast<int32_t*>(su.scratch + NA_PART_O_BYTES + NA_PART_ML_BYTES);
   // The counters must start at zero; the array keeps whatever the last call left.
-  e = cudaMemsetAsync(count, 0, (size_t)n_seq * d.kv_heads * sizeof(int32_t), s);
+  cudaError_t e = cudaMemsetAsync(count, 0, (size_t)n_seq * d.kv_heads * sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
   const float scale = LOG2E / sqrtf((float)d.head_dim);
-  attn_decode_noalloc_kernel<T, D><<<grid, NA_THREADS, smem, s>>>(
+  attn_decode_noalloc_kernel<T, D><<<grid, NA_THREADS, NaCfg<T, D>::SMEM, s>>>(
       d, layer, static_cast<const T*>(q), static_cast<T*>(out), scale, n_seq, cs, part_o,
       part_ml, count);
   return cudaGetLastError();
@@ -398,24 +464,13 @@ cudaError_t launch_typed(const Dev& d, int layer, const void* q, void* out, int 
 
 int noalloc_max_pairs() { return NA_MAX_PAIRS; }
 
-// Chunks per session: about four items per resident CTA over the call, limited by
-// the static scratch and by NA_MAX_CHUNKS.
-int noalloc_chunks(const Dev& d, int n_seq) {
-  const int pairs = n_seq * d.kv_heads;
-  int cs = std::max(1, 4 * 3 * 152 / std::max(1, pairs));
-  cs = std::min(cs, NA_MAX_CHUNKS);
-  cs = std::min(cs, NA_MAX_SLOTS / std::max(1, pairs));
-  return std::max(1, cs);
-}
-
 cudaError_t launch_attn_decode_noalloc(const Dev& d, int layer, const void* q, void* out,
-                                       int n_seq, int cs, cudaStream_t s) {
-  void* scratch = nullptr;
-  cudaError_t e = scratch_address(&scratch);
+                                       int n_seq, cudaStream_t s) {
+  NaSetup su;
+  cudaError_t e = setup_for_current_context(&su);
   if (e != cudaSuccess) return e;
-  uint8_t* sp = static_cast<uint8_t*>(scratch);
-  if (d.esz == 2) return launch_typed<__nv_bfloat16, 128>(d, layer, q, out, n_seq, cs, sp, s);
-  return launch_typed<float, 64>(d, layer, q, out, n_seq, cs, sp, s);
+  if (d.esz == 2) return launch_typed<__nv_bfloat16, 128>(d, layer, q, out, n_seq, su, s);
+  return launch_typed<float, 64>(d, layer, q, out, n_seq, su, s);
 }
 
 }  // namespace kvc

@@ -221,6 +221,13 @@ class Driver:
                 on_evict(st)
         return launches
 
+    def release(self, sessions) -> None:
+        """End sessions (kvc_release): their positions start over at 0; later steps feed
+        them the rest of their scripts."""
+        self.cache.release(np.asarray(sessions, dtype=np.int32))
+        for s in sessions:
+            self.pos[s] = 0
+
     def fast_forward(self, n_steps: int) -> None:
         """Advance the cache state without attention (attention does not change state)."""
         for _ in range(n_steps):

@@ -236,6 +236,52 @@ def test_single_session_full_size_metadata_and_sampled_attention():
     assert st["peak_resident"] > 4096
 
 
+@pytest.mark.parametrize("budget", [8192, 0])
+def test_single_session_full_size_table3_budgets(budget):
+    """Table 3's other budgets on the full-size single-session workload (32 layers, 600
+    units): B = 8K and the B = 0 floor.  Every evict bit-exact, peak resident count
+    included (End and Peak of Table 3 are the device's resident and peak_resident at the
+    end); attention sampled."""
+    ls, _ = _lockstep(S.SINGLE_BF16.with_(budget=budget))
+    last = len(ls.drv.sched) - 1
+    samples = {300, last}
+    for step in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda st, kind, i, layer: st in samples and layer == 0
+                    and i in (0, 1))
+    st = ls.drv.cache.export_state(0)
+    ref = ls.orc.state(0)
+    assert (st["resident"], st["peak_resident"]) == (ref["resident"], ref["peak_resident"])
+    if budget > 0:
+        assert st["resident"] <= budget < st["peak_resident"]
+    else:
+        assert all(t in (2, 3) or u > ref["unit_cur"] - S.SINGLE_BF16.window
+                   for t, u in zip(st["type"], st["unit"]))
+    assert ls.n_compared >= 4
+
+
+@pytest.mark.parametrize("policy", ["unit", "position", "sink_recent"])
+def test_release_and_reuse(policy):
+    """kvc_release ends sessions mid-run; fed the rest of their scripts from position 0 they
+    evict as fresh sessions under the same policy.  Every state bit-exact after the release
+    and after every evict, every attention output compared."""
+    w = S.SINGLE_BF16.with_(layers=2, n_sessions=3, budget=60, window=1, seed=31,
+                            turn_period=9, turn_jitter=1, policy=policy, sink=3, recent=30)
+    ls, _ = _lockstep(w, n_units=36)
+    for _ in range(15):
+        ls.run_step(attn_pred=lambda *a: True)
+    free0, _ = ls.drv.cache.device_status()
+    held = sum(len(ls.orc.layout[s].hist_pages) + len(ls.orc.layout[s].live_pages)
+               for s in (0, 2))
+    ls.release([0, 2])
+    free1, err = ls.drv.cache.device_status()
+    assert err == 0 and free1 == free0 + held
+    for _ in range(len(ls.drv.sched) - 15):
+        ls.run_step(attn_pred=lambda *a: True)
+    for s in (0, 2):
+        assert ls.drv.cache.export_state(s)["n_evicted"] > 0
+    assert ls.n_compared > 100
+
+
 def test_single_session_unbounded_full_size():
     """No-eviction run of the single-session workload (B = infinity): every evict is a
     no-op checked bit-exact, the cache grows to every fed position (about 13.7K), and
@@ -283,24 +329,104 @@ def test_stress_shard(budget, window):
     assert ls.n_compared >= 16
 
 
+def _sms():
+    return torch.cuda.get_device_properties(0).multi_processor_count
+
+
+def _decode_tier(n_seq, kv_heads):
+    """Decode kernel the library dispatches for a call of n_seq sessions: the 16-warp pair
+    split (one CTA per SM, tensor-core pages) while every (session, KV head) pair gets two
+    slices, the 4-warp pair split while it gets three of the three CTAs per SM, else
+    stream-K."""
+    pairs = n_seq * kv_heads
+    if 2 * pairs <= _sms():
+        return "split16"
+    if 3 * pairs <= 3 * _sms():
+        return "split4"
+    return "streamk"
+
+
+def test_decode_4warp_tier_at_full_budget():
+    """Decode calls of 10-19 sessions (the 4-warp pair split on 152 SMs) at full budget,
+    every output of every session compared with the oracle: the first two natural decode
+    rounds of that size in a step of a 19-session shard of the 64-session workload at its
+    steady state, then calls of exactly 10, 12, 16 and 19 sessions (one transcript token
+    each)."""
+    w = S.BATCH64_BF16
+    scripts = S.workload_scripts(w)
+    shard = sorted(scripts, key=lambda sc: sc.offset)[:19]
+    drv = Driver(w, shard)
+    ls = Lockstep(drv, w)
+    steady = S.steady_state_step(w, shard)
+    for _ in range(steady):
+        ls.run_step(check_state=False)
+    tiers = {}
+    picked = []
+
+    def select(step, c, i, layer):
+        if c.kind != "decode" or layer != 0:
+            return None
+        tier = _decode_tier(len(c.sessions), w.kv_heads)
+        if tier != "split4" or len(picked) >= 2:
+            return None
+        picked.append(len(c.sessions))
+        tiers.setdefault(tier, set()).add(len(c.sessions))
+        return "all"
+
+    ls.run_step(select=select)
+    for n in (10, 12, 16, 19):
+        ls.decode_call([sc.session for sc in shard[:n]], layers=(0, 31) if n == 10 else (0,))
+        tiers.setdefault(_decode_tier(n, w.kv_heads), set()).add(n)
+    for sc in shard:
+        st = drv.cache.export_state(sc.session)
+        assert st["resident"] >= 4000 and st["n_evicted"] > 0
+    if _sms() == 152:
+        assert {10, 12, 16, 19} <= tiers["split4"]
+        assert len(picked) == 2
+    assert ls.n_compared >= 10 * 2 + 12 + 16 + 19
+
+
 def test_batch64_sampled_at_full_size():
-    """64 sessions, offsets U{0..300}: state of every session bit-exact at sampled steps;
-    attention of sampled sessions/layers in the launch configuration of the benchmark."""
+    """64 sessions, offsets U{0..300}, run through the benchmark's timed window (its 20
+    steps from the steady state): the state of every session bit-exact at sampled steps and
+    after every evict of the window; attention in the benchmark's launch configuration at
+    three steps of the window: the prefill call and the first decode round of each kernel
+    tier present (stream-K for >= 20 sessions, the 4-warp pair split for 10-19, the
+    16-warp tensor-core pair split for <= 9, and a one-session round)."""
     w = S.BATCH64_BF16
     scripts = S.workload_scripts(w)
     drv = Driver(w, scripts)
     ls = Lockstep(drv, w)
-    stop = S.steady_state_step(w, scripts) + 3
-    check = set(range(0, stop, 97)) | {stop - 1}
+    start = S.steady_state_step(w, scripts)
+    stop = start + 20
+    check = set(range(0, start, 97))
+    sampled = {start: 0, start + 9: 13, stop - 1: 31}   # step -> layer compared
+    seen = set()
+
+    def select(step, c, i, layer):
+        if sampled.get(step) != layer:
+            return None
+        if c.kind == "prefill":
+            return {0, 21, 42, 63}
+        n = len(c.sessions)
+        tier = "one" if n == 1 else _decode_tier(n, w.kv_heads)
+        if (tier, step) in seen:
+            return None
+        seen.add((tier, step))
+        stride = {"streamk": 16, "split4": 5, "split16": 3, "one": 1}[tier]
+        return {int(x) for x in c.sessions[::stride]}
+
     for step in range(stop):
-        if step in check or step >= stop - 3:
-            ls.run_step(attn_pred=lambda st, kind, i, layer: st >= stop - 2 and
-                        layer in (0, 13, 31) and i in (0, 1, 4),
-                        session_pred=lambda s: s % 21 == 0)
+        if step >= start or step in check:
+            ls.run_step(select=select)
         else:
-            # Oracle replays the policy without comparing every state.
-            ls.run_step(attn_pred=None, check_state=False)
-    assert ls.n_compared >= 12
+            # The oracle replays the policy without comparing every state.
+            ls.run_step(check_state=False)
+    tiers = {t for t, _ in seen}
+    assert {"streamk", "split16"} <= tiers
+    if _sms() == 152:
+        assert "split4" in tiers
+    assert ls.n_compared >= 30
 
 
 def test_compaction_is_a_pure_move():

@@ -4,7 +4,8 @@ while they decode (a real-time loop that must not stall on the device
 synchronisation an allocation can cause, or an application whose device memory
 belongs to another framework).  It must give the same result as
 kvc_attn_decode, within the tolerance of the attention parity tests, on calls
-made one after another (the array keeps the previous call's contents).
+made one after another (the array keeps the previous call's contents), and
+match the CPU oracle as the other decode paths do.
 
 This file is named so that pytest collects it last.
 """
@@ -17,7 +18,7 @@ torch = pytest.importorskip("torch")
 if not torch.cuda.is_available():
     pytest.skip("needs a CUDA GPU", allow_module_level=True)
 
-from harness import assert_close  # noqa: E402
+from harness import Lockstep, assert_close  # noqa: E402
 
 pytestmark = pytest.mark.gpu
 
@@ -30,58 +31,86 @@ def built():
     gpu.build()
 
 
-def _driver(w, units):
+def _lockstep(w, units):
     from synth import script as S
     from synth.driver import Driver
     scripts = S.workload_scripts(w)
     for sc in scripts:
         sc.n_transcript = sc.n_transcript[:units]
         sc.n_text = sc.n_text[:units]
-    return Driver(w, scripts)
+    return Lockstep(Driver(w, scripts), w)
 
 
 def _decode_both(drv, c, layer):
-    """Existing entry point, then the no-allocation one, on the same queries."""
+    """Existing entry point into a scratch buffer, then the no-allocation one into the
+    call's output buffer, on the same queries."""
     lib, ctx = drv.cache.lib, drv.cache.ctx
     stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
     ref = torch.empty_like(c.out)
-    got = torch.full_like(c.out, float("nan"))
+    c.out.fill_(float("nan"))
     assert lib.kvc_attn_decode(ctx, layer, c.q[layer].data_ptr(), ref.data_ptr(), stream) == 0
-    rc = lib.kvc_attn_decode_noalloc(ctx, layer, c.q[layer].data_ptr(), got.data_ptr(), stream)
+    rc = lib.kvc_attn_decode_noalloc(ctx, layer, c.q[layer].data_ptr(), c.out.data_ptr(), stream)
     assert rc == 0, lib.kvc_last_error()
     torch.cuda.synchronize()
-    return got.float().cpu().numpy(), ref.float().cpu().numpy()
+    return c.out.float().cpu().numpy(), ref.float().cpu().numpy()
 
 
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
-def test_noalloc_decode_matches_decode_on_consecutive_calls(dtype):
-    from synth import script as S
-    if dtype == "bf16":
-        w = S.SINGLE_BF16.with_(layers=2, n_sessions=5, offset_max=3, budget=150, window=2,
-                                seed=21, turn_period=7, turn_jitter=1)
-    else:
-        w = S.TINY_F32.with_(n_sessions=3, offset_max=2, budget=120, window=2, seed=22)
-    drv = _driver(w, 18)
-    compared = 0
+def _run(ls, dtype, layers, oracle_pred):
+    """Every step of the lockstep run; each decode call answered by both entry points at
+    `layers` (two calls in a row), compared with each other, and the decode calls that
+    oracle_pred(index of the decode call, call) selects also compared with the oracle."""
+    drv = ls.drv
+    compared, n_dec = 0, 0
     for _ in range(len(drv.sched)):
         st = drv.prepare_step()
         for c in st.calls:
             drv.cache.append_chunk(c.sessions, c.cu, c.types, c.k, c.v)
+            ls.on_append(c)
             if c.kind != "decode":
                 continue
-            # Two calls in a row (two layers, or the same layer twice), each compared.
-            for layer in ([0, w.layers - 1] if w.layers > 1 else [0, 0]):
+            for layer in layers:
                 got, ref = _decode_both(drv, c, layer)
                 assert np.isfinite(got).all()
                 assert_close(got, ref, dtype, f"step {st.index} layer {layer}")
+                if oracle_pred(n_dec, c):
+                    ls.compare_call(c, layer, None, f"no-allocation step {st.index}")
                 compared += 1
+            n_dec += 1
         if st.evict_sessions is not None:
             drv.cache.evict(st.evict_sessions)
-    assert compared >= 20
+            ls.orc.evict(st.evict_sessions.tolist())
+    return compared
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_noalloc_decode_matches_decode_and_oracle_on_consecutive_calls(dtype):
+    from synth import script as S
+    if dtype == "bf16":
+        w = S.SINGLE_BF16.with_(layers=2, n_sessions=5, offset_max=3, budget=150, window=2,
+                                seed=21, turn_period=7, turn_jitter=1)
+        layers = [0, 1]
+    else:
+        w = S.TINY_F32.with_(n_sessions=3, offset_max=2, budget=120, window=2, seed=22)
+        layers = [0, 0]
+    ls = _lockstep(w, 18)
+    assert _run(ls, dtype, layers, lambda i, c: i % 3 == 0) >= 20
+    assert ls.n_compared >= 20
+
+
+def test_noalloc_decode_single_chunk_calls():
+    """Decode rounds of all 120 sessions: 120 x 8 KV heads = 960 (session, KV head) pairs,
+    more than four work items per resident CTA (3 x 152), so every pair is one chunk and
+    its CTA writes the output directly (no partial state, no merge).  Those calls are
+    compared with the oracle; the smaller rounds with the workspace entry point."""
+    from synth import script as S
+    w = S.SINGLE_BF16.with_(layers=1, n_sessions=120, budget=-1, seed=23, turns=False)
+    ls = _lockstep(w, 3)
+    assert _run(ls, "bf16", [0, 0], lambda i, c: len(c.sessions) == 120) >= 4
+    assert ls.n_compared >= 4 * 120
 
 
 def test_noalloc_decode_rejects_calls_beyond_its_scratch():
-    from paper_2609_31224_gb300 import KVCache, KvcError
+    from paper_2609_31224_gb300 import KVCache
     # 65 sessions x 64 kv heads = 4160 (session, kv-head) pairs > 4096.
     c = KVCache(n_sessions=65, layers=1, q_heads=256, kv_heads=64, head_dim=128, budget=-1,
                 window=0, dtype="bf16", n_pages=80, max_pages_per_session=2, max_positions=8,
