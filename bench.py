@@ -43,7 +43,7 @@ UNIT = "audio-s/s"
 DECODE_TRAFFIC_RATIO = 410.93 / 403.97
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "f36ab38985938043022c24377366d8409783aba1dc77a03b1f3530905e77c25c"
+DECODE_TRAFFIC_SHA256 = "d3af0d34fdb37240047f3343c6c9fc6978385df2b1b56cf853199aeee0a732a0"
 
 
 def decode_traffic(alg_bytes_per_launch):

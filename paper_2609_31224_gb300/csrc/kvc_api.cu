@@ -7,7 +7,7 @@
 #include <string>
 #include <vector>
 
-#include "kvc_internal.cuh"
+#include "kvc_launch.cuh"
 
 using namespace kvc;
 
@@ -359,12 +359,13 @@ int kvc_append_chunk(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, const i
   AppendArgs a;
   a.n_seq = n_seq;
   a.total = total;
-  a.pf_target = ctx->pf_target;
+  // Only the binary32 prefill kernel reads the per-session chunk list.
+  a.pf_target = ctx->d.esz == 4 ? ctx->pf_target : 0;
   a.pf_min_blocks = 4;
   for (int i = 0; i < n_seq; ++i) a.sessions[i] = h_sessions[i];
   for (int i = 0; i <= n_seq; ++i) a.cu[i] = h_cu_tokens[i];
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  KVC_CUDA(launch_append(ctx->d, a, d_types, d_k, d_v, s));
+  KVC_CUDA(launch_append(ctx->d, a, d_types, d_k, d_v, single, s));
   for (int i = 0; i < n_seq; ++i) {
     const int sid = h_sessions[i];
     const int t = h_cu_tokens[i + 1] - h_cu_tokens[i];

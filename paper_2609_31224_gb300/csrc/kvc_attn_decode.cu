@@ -23,7 +23,7 @@
 // would repeat the tag) use the acquire-release arrival.
 #include <cstring>
 
-#include "kvc_internal.cuh"
+#include "kvc_launch.cuh"
 
 // Shape constants of the CUDA-core loop are unused by the tensor-core shapes.
 #pragma nv_diag_suppress 177
@@ -807,6 +807,34 @@ __device__ void publish_tagged(const Dev& d, const Smem<C>& sm, int slot, uint32
   if (tid < 2 * G) st_tagged(ts + G * C::D + tid, tag, sm.r_ml[tid]);
 }
 
+// Re-read, all in one pass, the words of w[] (loaded from p(i)) whose tag is not
+// yet `tag`, until every word carries it: the stores of the other CTAs were issued
+// before their arrivals and land within a round trip or two, so reloading every
+// stale word at once costs about one round trip instead of one per stale word.
+// Gives up (KVC_DERR_WAIT) after WAIT_LIMIT_CYCLES, keeping the stale values.
+template <int N, typename PtrFn>
+__device__ inline void settle_tagged(const Dev& d, unsigned long long (&w)[N], uint32_t tag,
+                                     PtrFn p) {
+  long long t0 = 0;
+  for (bool first = true;; first = false) {
+    bool stale = false;
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+      if ((uint32_t)(w[i] >> 32) != tag) {
+        w[i] = ld_tagged(p(i));
+        stale = true;
+      }
+    }
+    if (!stale) return;
+    if (first) {
+      t0 = clock64();
+    } else if (clock64() - t0 > WAIT_LIMIT_CYCLES) {
+      set_error(d, KVC_DERR_WAIT);
+      return;
+    }
+  }
+}
+
 // merge_parts over the tagged states of slots slot0 .. slot0 + nch - 1 of this
 // launch (tag): every load is a single 64-bit word whose tag says whether its
 // store has landed.
@@ -820,36 +848,35 @@ __device__ void merge_tagged(const Dev& d, const Smem<C>& sm, int nch, int slot0
   constexpr int CH = 24 / EPT > 0 ? 24 / EPT : 1;
   const unsigned long long* base = tagged_slot<C>(d, slot0);
   const unsigned long long filler = (unsigned long long)tag << 32;  // 0.0f, current tag
-  unsigned long long a[CH][EPT];
+  unsigned long long a[CH * EPT];
+  auto word = [&](int c0, int j) -> const unsigned long long* {
+    return base + (size_t)(c0 + j / EPT) * TW + tid + (j % EPT) * C::THREADS;
+  };
   auto load_batch = [&](int c0) {
 #pragma unroll
-    for (int i = 0; i < CH; ++i)
-#pragma unroll
-      for (int t = 0; t < EPT; ++t) {
-        const int e = tid + t * C::THREADS;
-        a[i][t] = (c0 + i < nch && e < G * D) ? ld_tagged(base + (size_t)(c0 + i) * TW + e)
-                                              : filler;
-      }
+    for (int j = 0; j < CH * EPT; ++j) {
+      const int e = tid + (j % EPT) * C::THREADS;
+      a[j] = (c0 + j / EPT < nch && e < G * D) ? ld_tagged(word(c0, j)) : filler;
+    }
   };
   load_batch(0);
   if (warp < G) {
     const int g = warp;
     constexpr int PL = MAX_PARTS / 32;
-    unsigned long long wm[PL], wl[PL];
+    unsigned long long wml[2 * PL];
+    auto ml_word = [&](int j) -> const unsigned long long* {
+      return base + (size_t)(lane + 32 * (j / 2)) * TW + G * D + 2 * g + (j % 2);
+    };
 #pragma unroll
-    for (int i = 0; i < PL; ++i) {
-      const int ch = lane + 32 * i;
-      const unsigned long long* p = base + (size_t)ch * TW + G * D + 2 * g;
-      wm[i] = ch < nch ? ld_tagged(p) : filler;
-      wl[i] = ch < nch ? ld_tagged(p + 1) : filler;
-    }
+    for (int j = 0; j < 2 * PL; ++j)
+      wml[j] = lane + 32 * (j / 2) < nch ? ld_tagged(ml_word(j)) : filler;
+    settle_tagged(d, wml, tag, ml_word);
     float m[PL], l[PL], M = -INFINITY;
 #pragma unroll
     for (int i = 0; i < PL; ++i) {
       const int ch = lane + 32 * i;
-      const unsigned long long* p = base + (size_t)ch * TW + G * D + 2 * g;
-      m[i] = ch < nch ? tagged_value(d, p, wm[i], tag) : -INFINITY;
-      l[i] = ch < nch ? tagged_value(d, p + 1, wl[i], tag) : 0.f;
+      m[i] = ch < nch ? __uint_as_float((uint32_t)wml[2 * i]) : -INFINITY;
+      l[i] = ch < nch ? __uint_as_float((uint32_t)wml[2 * i + 1]) : 0.f;
       M = fmaxf(M, m[i]);
     }
 #pragma unroll
@@ -872,6 +899,7 @@ __device__ void merge_tagged(const Dev& d, const Smem<C>& sm, int nch, int slot0
 #pragma unroll
   for (int t = 0; t < EPT; ++t) O[t] = 0.f;
   for (int c0 = 0;;) {
+    settle_tagged(d, a, tag, [&](int j) { return word(c0, j); });
 #pragma unroll
     for (int i = 0; i < CH; ++i) {
       if (c0 + i >= nch) break;
@@ -879,8 +907,7 @@ __device__ void merge_tagged(const Dev& d, const Smem<C>& sm, int nch, int slot0
       for (int t = 0; t < EPT; ++t) {
         const int e = tid + t * C::THREADS;
         if (e < G * D)
-          O[t] += tagged_value(d, base + (size_t)(c0 + i) * TW + e, a[i][t], tag) *
-                  sm.s_scale[(c0 + i) * G + e / D];
+          O[t] += __uint_as_float((uint32_t)a[i * EPT + t]) * sm.s_scale[(c0 + i) * G + e / D];
       }
     }
     c0 += CH;

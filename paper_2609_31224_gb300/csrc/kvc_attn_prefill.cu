@@ -12,7 +12,7 @@
 
 #include <algorithm>
 
-#include "kvc_internal.cuh"
+#include "kvc_launch.cuh"
 
 namespace kvc {
 

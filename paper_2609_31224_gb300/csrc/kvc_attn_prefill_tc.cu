@@ -24,7 +24,7 @@
 // All waits are bounded; a timeout records KVC_DERR_WAIT and the CTA stops.
 #include <cuda.h>
 
-#include "kvc_internal.cuh"
+#include "kvc_launch.cuh"
 
 namespace kvc {
 

@@ -264,22 +264,6 @@ __device__ inline unsigned long long ld_tagged(const unsigned long long* p) {
   asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
   return w;
 }
-// Value of word w (loaded from p) once its tag is `tag`; 0 with KVC_DERR_WAIT
-// recorded if the store does not show up within WAIT_LIMIT_CYCLES.
-__device__ inline float tagged_value(const Dev& d, const unsigned long long* p,
-                                     unsigned long long w, uint32_t tag) {
-  if ((uint32_t)(w >> 32) != tag) {
-    const long long t0 = clock64();
-    do {
-      if (clock64() - t0 > WAIT_LIMIT_CYCLES) {
-        set_error(d, KVC_DERR_WAIT);
-        return 0.f;
-      }
-      w = ld_tagged(p);
-    } while ((uint32_t)(w >> 32) != tag);
-  }
-  return __uint_as_float((uint32_t)w);
-}
 __device__ inline bool arrive_relaxed(int* counter, int parts) {
   int old;
   asm volatile("atom.relaxed.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(counter) : "memory");
@@ -427,54 +411,5 @@ __device__ inline float to_float<__nv_bfloat16>(__nv_bfloat16 x) {
 __device__ inline float exp2_safe(float x, float m) {
   return (m == -INFINITY) ? 0.f : exp2f(x - m);
 }
-
-// ---------------------------------------------------------------------------
-// Launchers (defined in the .cu files).
-// ---------------------------------------------------------------------------
-struct AppendArgs {
-  int32_t n_seq;
-  int32_t total;
-  int32_t pf_target;       // desired item count of the binary32 prefill's chunk list
-  int32_t pf_min_blocks;
-  int32_t sessions[MAX_SEQ];
-  int32_t cu[MAX_SEQ + 1];
-};
-
-struct SeqArgs {
-  int32_t n_seq;
-  int32_t sessions[MAX_SEQ];
-};
-
-cudaError_t launch_init(const Dev& d, double rope_base, cudaStream_t s);
-cudaError_t launch_append(const Dev& d, const AppendArgs& a, const uint8_t* types, const void* k,
-                          const void* v, cudaStream_t s);
-cudaError_t launch_append_layers(const Dev& d, int total, int layer0, int n_layers, const void* k,
-                                 const void* v, cudaStream_t s);
-cudaError_t launch_evict(const Dev& d, const SeqArgs& a, int64_t* resident_out, cudaStream_t s);
-cudaError_t launch_release(const Dev& d, const SeqArgs& a, cudaStream_t s);
-cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_out, void* k_out,
-                              void* v_out, int32_t* count, cudaStream_t s);
-// new_k / new_v (optional): the fused per-layer write of the new tokens' K/V.
-// epoch: tag of this launch's partial states (nonzero, never reused while tags
-// of it may remain in the slots); 0 selects the fenced arrival instead.
-cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               bool pdl, cudaStream_t s, uint32_t epoch,
-                               const void* new_k = nullptr, const void* new_v = nullptr);
-cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                                int max_t, bool pdl, cudaStream_t s);
-cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,
-                                   const CUtensorMap& hi, const void* q, void* out, int grid,
-                                   bool pdl, cudaStream_t s);
-const void* prefill_tc_kernel_ptr();
-// Two 2-D views of the bfloat16 pool as rows of 128 elements (columns 0-63 and
-// 64-127), 16-row boxes, 128-byte swizzle; cached per pool.  False if the driver
-// entry point is missing or the encoding fails.
-bool pool_tensor_maps(const Dev& d, CUtensorMap* lo, CUtensorMap* hi);
-int prefill_tc_smem();
-int prefill_tc_threads();
-int noalloc_max_pairs();
-cudaError_t launch_attn_decode_noalloc(const Dev& d, int layer, const void* q, void* out,
-                                       int n_seq, cudaStream_t s);
-int prefill_grid_ctas(const Dev& d);
 
 }  // namespace kvc

@@ -6,7 +6,7 @@
 // session order then token order (append) or session order (evict: all
 // sessions' compacted-region pages are allocated before any live page is
 // freed).  This makes page tables a deterministic function of the calls.
-#include "kvc_internal.cuh"
+#include "kvc_launch.cuh"
 
 namespace kvc {
 
@@ -321,8 +321,12 @@ __global__ void __launch_bounds__(META_THREADS) append_plan_kernel(Dev d, Append
     }
     __syncthreads();
   }
-  build_worklist(d, n_seq, nb, a.pf_target, a.pf_min_blocks, d.max_pf_items, d.pf_items, s_warp,
-                 &s_total_pf);
+  if (a.pf_target > 0) {
+    build_worklist(d, n_seq, nb, a.pf_target, a.pf_min_blocks, d.max_pf_items, d.pf_items,
+                   s_warp, &s_total_pf);
+  } else if (i == 0) {
+    s_total_pf = 0;
+  }
   if (i == 0) {
     d.g->n_seq = n_seq;
     d.g->total_tokens = a.total;
@@ -330,6 +334,14 @@ __global__ void __launch_bounds__(META_THREADS) append_plan_kernel(Dev d, Append
     d.g->n_pf_items = s_total_pf;
     d.g->pages_used += total_need;
   }
+}
+
+// Rotate-half RoPE of one pair (x1, x2) = (k[j], k[j + D/2]) with (cos, sin) of
+// the position's angle for dim j, in binary32 on the binary32 table.  Every K
+// writer uses this one expression, so stored keys do not depend on the path.
+__device__ inline void rope_pair(float x1, float x2, float2 c, float& y1, float& y2) {
+  y1 = fmaf(x1, c.x, -x2 * c.y);
+  y2 = fmaf(x2, c.x, x1 * c.y);
 }
 
 // Append, part 2: K rotated at its position (rotate-half, binary32 math on
@@ -353,9 +365,8 @@ __global__ void __launch_bounds__(256) append_kv_kernel(Dev d, int total, int la
     const int h = idx / half, j = idx % half;
     const float x1 = to_float<T>(kin[h * D + j]);
     const float x2 = to_float<T>(kin[h * D + j + half]);
-    const float2 c = cs[j];
-    const float y1 = fmaf(x1, c.x, -x2 * c.y);
-    const float y2 = fmaf(x2, c.x, x1 * c.y);
+    float y1, y2;
+    rope_pair(x1, x2, cs[j], y1, y2);
     T* dst = pool + pool_offset_elems(d, page, l, 0, h, slot);
     dst[j] = from_float<T>(y1);
     dst[j + half] = from_float<T>(y2);
@@ -365,6 +376,200 @@ __global__ void __launch_bounds__(256) append_kv_kernel(Dev d, int total, int la
     const int h = (idx * vec) / D, j = (idx * vec) % D;
     const uint4 x = *reinterpret_cast<const uint4*>(vin + h * D + j);
     *reinterpret_cast<uint4*>(pool + pool_offset_elems(d, page, l, 1, h, slot) + j) = x;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Append of exactly one token per session (the decode rounds): thread i plans
+// session i of the call (page demand, lowest-free allocation in call order,
+// position, unit, slot tags, state, the attention calls' work split); when k and
+// v are given the CTA then writes the tokens' rotated K and V of every layer.
+// Same state, tags and stored bytes as the general plan kernel followed by
+// append_kv_kernel.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(META_THREADS) append_single_kernel(Dev d, AppendArgs a,
+                                                                     const uint8_t* types,
+                                                                     const T* k, const T* v) {
+  __shared__ int s_warp[33];
+  __shared__ int s_bad, s_total_pf;
+  __shared__ int s_gs[MAX_SEQ], s_pos[MAX_SEQ];
+  const int i = threadIdx.x;
+  const int n_seq = a.n_seq;
+  const int mpps = d.max_pages_per_session;
+  if (i == 0) s_bad = 0;
+  __syncthreads();
+
+  int sid = 0, need = 0, ty = 0, page = 0;
+  SessState st = {};
+  if (i < n_seq) {
+    sid = a.sessions[i];
+    st = d.sess[sid];
+    ty = (int)types[i];
+    const int tail = st.live_head + st.n_live;
+    need = (tail + PS) / PS - st.n_live_pages;
+    if (need < 0 || need > 1 || st.n_live_pages + need > mpps)
+      atomicOr(&s_bad, KVC_DERR_PAGE_TABLE);
+    if (st.pos_next + 1 > d.max_positions) atomicOr(&s_bad, KVC_DERR_POSITION);
+    if (need == 0) page = d.live_pt[(size_t)sid * mpps + tail / PS];
+  }
+  __syncthreads();
+  if (s_bad) {
+    if (i == 0) {
+      set_error(d, s_bad);
+      abandon_append(d);
+    }
+    return;
+  }
+  int total_need;
+  const int off = block_exclusive_scan(need, &total_need, s_warp);
+  if (total_need > 0 && (total_need > d.max_alloc || !block_alloc_lowest(d, total_need, s_warp))) {
+    if (i == 0) {
+      set_error(d, KVC_DERR_POOL);
+      abandon_append(d);
+    }
+    return;
+  }
+  int nb = 0;
+  SeqInfo si = {};
+  if (i < n_seq) {
+    const int tail = st.live_head + st.n_live;
+    if (need) {
+      page = d.alloc_list[off];
+      d.live_pt[(size_t)sid * mpps + st.n_live_pages] = page;
+    }
+    const int gs = page * PS + tail % PS;
+    const int unit = st.unit_cur + ((ty & KVC_UNIT_BEGIN) ? 1 : 0);
+    d.meta_pos[gs] = st.pos_next;
+    d.meta_unit[gs] = unit;
+    d.meta_type[gs] = (uint8_t)(ty & TYPE_MASK);
+    d.tok_slot[i] = gs;
+    d.tok_pos[i] = st.pos_next;
+    s_gs[i] = gs;
+    s_pos[i] = st.pos_next;
+    SessState s1 = st;
+    s1.pos_next = st.pos_next + 1;
+    s1.unit_cur = unit;
+    s1.n_live = st.n_live + 1;
+    s1.last_chunk = 1;
+    s1.n_live_pages = st.n_live_pages + need;
+    s1.peak_resident = max(st.peak_resident, s1.n_hist + s1.n_live);
+    d.sess[sid] = s1;
+    nb = s1.n_hist_pages + s1.n_live_pages;
+    si.sid = sid;
+    si.t = 1;
+    si.q_row0 = i;
+    si.pos_first = st.pos_next;
+    si.n_hist = s1.n_hist;
+    si.n_hist_pages = s1.n_hist_pages;
+    si.live_head = s1.live_head;
+    si.n_live = s1.n_live;
+    si.n_blocks = nb;
+  }
+  // Split-K work of the attention calls (as in append_plan_kernel).
+  int total_units;
+  const int ubase = block_exclusive_scan(i < n_seq ? nb * d.kv_heads : 0, &total_units, s_warp);
+  const int nb_max = block_max(i < n_seq ? nb : 0, s_warp);
+  if (i < n_seq) {
+    si.unit_base = ubase;
+    d.seq[i] = si;
+  }
+  __syncthreads();
+  s_total_pf = 0;
+  if (a.pf_target > 0)
+    build_worklist(d, n_seq, nb, a.pf_target, a.pf_min_blocks, d.max_pf_items, d.pf_items,
+                   s_warp, &s_total_pf);
+  if (i == 0) {
+    d.g->n_seq = n_seq;
+    d.g->total_tokens = n_seq;
+    d.g->n_units = total_units;
+    d.g->nb_max = nb_max;
+    d.g->n_pf_items = s_total_pf;
+    d.g->pages_used += total_need;
+  }
+  if (k == nullptr) return;
+  __syncthreads();
+  // K rotated at the token's position and V, every layer and head: one 16-byte chunk
+  // of the first half of a K row with its rotate-half partner per K item, one 16-byte
+  // chunk of V per V item; K/V input layout [L][n_seq][Hkv][D].  Each thread loads U
+  // items before it stores any, so their loads are in flight together.
+  constexpr int VEC = 16 / sizeof(T), U = 4;
+  const int D = d.head_dim, half = D / 2, H = d.kv_heads, L = d.layers;
+  T* pool = reinterpret_cast<T*>(d.pool);
+  const int kc = half / VEC, vc = D / VEC;
+  const int n_k = n_seq * L * H * kc, n_v = n_seq * L * H * vc;
+  auto decompose = [&](int idx, int per, int& c, int& h, int& q, int& l) {
+    c = idx % per;
+    int r = idx / per;
+    h = r % H;
+    r /= H;
+    q = r % n_seq;
+    l = r / n_seq;
+  };
+  for (int base = i; base < n_k; base += U * META_THREADS) {
+    uint4 wa[U], wb[U];
+    float4 cs[U][VEC / 2];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int idx = base + u * META_THREADS;
+      if (idx < n_k) {
+        int c, h, q, l;
+        decompose(idx, kc, c, h, q, l);
+        const T* kin = k + (((size_t)l * n_seq + q) * H + h) * D + c * VEC;
+        wa[u] = *reinterpret_cast<const uint4*>(kin);
+        wb[u] = *reinterpret_cast<const uint4*>(kin + half);
+        const float4* t4 = reinterpret_cast<const float4*>(d.rope + (size_t)s_pos[q] * half + c * VEC);
+#pragma unroll
+        for (int e = 0; e < VEC / 2; ++e) cs[u][e] = t4[e];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int idx = base + u * META_THREADS;
+      if (idx >= n_k) break;
+      int c, h, q, l;
+      decompose(idx, kc, c, h, q, l);
+      const T* xa = reinterpret_cast<const T*>(&wa[u]);
+      const T* xb = reinterpret_cast<const T*>(&wb[u]);
+      uint4 ya, yb;
+      T* pa = reinterpret_cast<T*>(&ya);
+      T* pb = reinterpret_cast<T*>(&yb);
+#pragma unroll
+      for (int e = 0; e < VEC; ++e) {
+        const float4 t = cs[u][e / 2];
+        const float2 ce = (e & 1) ? make_float2(t.z, t.w) : make_float2(t.x, t.y);
+        float y1, y2;
+        rope_pair(to_float<T>(xa[e]), to_float<T>(xb[e]), ce, y1, y2);
+        pa[e] = from_float<T>(y1);
+        pb[e] = from_float<T>(y2);
+      }
+      const int gs = s_gs[q];
+      T* dst = pool + pool_offset_elems(d, gs / PS, l, 0, h, gs % PS) + c * VEC;
+      *reinterpret_cast<uint4*>(dst) = ya;
+      *reinterpret_cast<uint4*>(dst + half) = yb;
+    }
+  }
+  for (int base = i; base < n_v; base += U * META_THREADS) {
+    uint4 x[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int idx = base + u * META_THREADS;
+      if (idx < n_v) {
+        int c, h, q, l;
+        decompose(idx, vc, c, h, q, l);
+        x[u] = *reinterpret_cast<const uint4*>(v + (((size_t)l * n_seq + q) * H + h) * D + c * VEC);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int idx = base + u * META_THREADS;
+      if (idx >= n_v) break;
+      int c, h, q, l;
+      decompose(idx, vc, c, h, q, l);
+      const int gs = s_gs[q];
+      *reinterpret_cast<uint4*>(pool + pool_offset_elems(d, gs / PS, l, 1, h, gs % PS) + c * VEC) =
+          x[u];
+    }
   }
 }
 
@@ -770,7 +975,23 @@ cudaError_t launch_init(const Dev& d, double rope_base, cudaStream_t s) {
 }
 
 cudaError_t launch_append(const Dev& d, const AppendArgs& a, const uint8_t* types, const void* k,
-                          const void* v, cudaStream_t s) {
+                          const void* v, bool single, cudaStream_t s) {
+  if (single) {
+    // One CTA writes the K/V rows only for a one-session call (a few hundred KiB at
+    // most); larger calls keep the plan in one CTA and spread the rows over
+    // append_kv_kernel's grid.
+    const bool fuse_kv = a.n_seq == 1;
+    if (d.esz == 2)
+      append_single_kernel<__nv_bfloat16><<<1, META_THREADS, 0, s>>>(
+          d, a, types, static_cast<const __nv_bfloat16*>(fuse_kv ? k : nullptr),
+          static_cast<const __nv_bfloat16*>(fuse_kv ? v : nullptr));
+    else
+      append_single_kernel<float><<<1, META_THREADS, 0, s>>>(
+          d, a, types, static_cast<const float*>(fuse_kv ? k : nullptr),
+          static_cast<const float*>(fuse_kv ? v : nullptr));
+    if (fuse_kv || k == nullptr) return cudaGetLastError();
+    return launch_append_layers(d, a.total, 0, d.layers, k, v, s);
+  }
   append_plan_kernel<<<1, META_THREADS, 0, s>>>(d, a, types);
   if (k == nullptr) return cudaGetLastError();  // plan only: layers follow one by one
   return launch_append_layers(d, a.total, 0, d.layers, k, v, s);

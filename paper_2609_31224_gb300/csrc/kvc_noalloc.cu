@@ -14,7 +14,7 @@
 #include <algorithm>
 #include <mutex>
 
-#include "kvc_internal.cuh"
+#include "kvc_launch.cuh"
 
 namespace kvc {
 
