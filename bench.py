@@ -38,12 +38,13 @@ UNIT = "audio-s/s"
 
 # DRAM bytes per algorithmic byte of the roofline kernel (reads + writes), from one
 # ncu capture of the stream-K kernel on the 24-session, two-layer reduced case:
-# 410.93 MB of traffic (406.82 MB read, 4.11 MB written) for a 403.97 MB launch.  Valid only while the decode sources
+# 410.69 MB of traffic (406.84 MB read, 3.85 MB written) for a 403.97 MB launch.  Valid only while the decode sources
 # hash to the version it was taken on; the roofline's traffic is null otherwise.
-DECODE_TRAFFIC_RATIO = 410.93 / 403.97
+DECODE_TRAFFIC_RATIO = 410.69 / 403.97
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
+                          "paper_2609_31224_gb300/csrc/kvc_decode_common.cuh",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "d3af0d34fdb37240047f3343c6c9fc6978385df2b1b56cf853199aeee0a732a0"
+DECODE_TRAFFIC_SHA256 = "827208e31cdde3946b24310eec0fba47957f0a4139e83994ba0fcce1a6e5529b"
 
 
 def decode_traffic(alg_bytes_per_launch):
@@ -552,6 +553,59 @@ def run_budget_sweep(n_sessions: int) -> dict:
             "sessions_per_budget": n_sessions, "rows": rows, "clocks": clk}
 
 
+# -- the stress workload at scale ------------------------------------------------------------
+def run_stress(budget: int, window: int, n_sessions: int, steps: int, warmup: int) -> dict:
+    """The stress workload (10-60 minute sessions, 5 % units without a segment, 2 % long
+    segments of 10-30 tokens) at one (B, W) grid point with `n_sessions` concurrent
+    sessions: the cache is brought (append + evict only) to the step where every session
+    is at its budget, then `warmup` and `steps` timed steps of the whole path (append,
+    every layer's attention, evict).  The scripts are cut after the last timed step, so
+    the pool is sized for the positions fed until then."""
+    import torch
+    from synth import script as S
+    from synth.driver import Driver
+    w = S.stress256(budget, window).with_(n_sessions=n_sessions)
+    scripts = S.workload_scripts(w)
+    start = S.steady_state_step(w, scripts)
+    keep = start + warmup + steps
+    for sc in scripts:
+        sc.n_transcript = sc.n_transcript[:keep]
+        sc.n_text = sc.n_text[:keep]
+    # Pool: each session's resident bound (budget or protected content, plus one unit) in
+    # pages, plus ten pages for partly filled pages and the eviction's transient.
+    from synth.driver import cache_sizing, resident_bound
+    sizing = cache_sizing(w, scripts)
+    sizing["n_pages"] = sum(resident_bound(w, sc)[0] // w.page_size + 10 for sc in scripts) + 16
+    drv = Driver(w, scripts, sizing=sizing)
+    drv.fast_forward(start)
+    for _ in range(warmup):
+        drv.run_step(drv.prepare_step())
+    timed = [drv.prepare_step() for _ in range(steps)]
+    torch.cuda.synchronize()
+    clocks = Clocks(torch.cuda.current_device())
+    clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    launches = 0
+    for st in timed:
+        launches += drv.run_step(st)
+    e1.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    audio_s = sum(len(st.pairs) for st in timed)
+    resident = [drv.cache.export_state(sc.session)["resident"] for sc in scripts[:8]]
+    return {"metric": METRIC, "value": audio_s / (ms / 1e3), "unit": UNIT, "steps": steps,
+            "warmup": warmup, "ms_per_step": ms / steps, "higher_is_better": True,
+            "dtype": w.dtype, "data": "synthetic (seeded SplitMix64 Irwin-Hall values, PCG64 "
+                                       "session scripts)",
+            "config": {"workload": w.name, "sessions": n_sessions, "budget": budget,
+                       "window": window, "timed_steps": [start + warmup, keep],
+                       "pool_pages": drv.sizing["n_pages"],
+                       "resident_first_sessions": resident},
+            "gpu_launches": launches, "clocks": clk}
+
+
 # -- the oracle on the host cores -----------------------------------------------------------------
 _BLAS_THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
 
@@ -696,6 +750,9 @@ def main():
                          "just before its attention")
     ap.add_argument("--budget-sweep", type=int, default=0, metavar="SESSIONS",
                     help="print the Table-3-shaped budget sweep over SESSIONS sessions and exit")
+    ap.add_argument("--stress", default=None, metavar="B,W[,N]",
+                    help="print one JSON line for the stress workload at budget B, window W "
+                         "with N concurrent sessions (default 256) and exit")
     ap.add_argument("--sessions", type=int, default=None,
                     help="reduced case for profiler captures (default: the full 64)")
     ap.add_argument("--layers", type=int, default=None,
@@ -727,6 +784,12 @@ def main():
     if args.budget_sweep:
         if rank == 0:
             print(json.dumps(run_budget_sweep(args.budget_sweep)))
+        return
+    if args.stress:
+        if rank == 0:
+            f = [int(x) for x in args.stress.split(",")]
+            print(json.dumps(run_stress(f[0], f[1], f[2] if len(f) > 2 else 256, args.steps,
+                                        args.warmup)))
         return
     out = run_ours(args, rank, world, local_rank)
     if rank == 0:

@@ -212,6 +212,19 @@ int kvc_evict(kvc_ctx* ctx, int n_seq, const int32_t* h_sessions, int64_t* d_res
 int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out,
                            void* stream);
 
+/* Chunked-prefill attention of one layer fused with that layer's K/V write (the
+ * per-layer order, after kvc_append_chunk without K/V; Sec. 3.1: a layer's keys
+ * and values of the unit's positions exist only once that layer has run): the
+ * chunk's K (rotated at its positions) and V of the layer are written into their
+ * slots and attended in the same call.  Same results and stored bytes as
+ * kvc_append_kv_layer followed by kvc_attn_prefill_chunk.  For bfloat16 the write
+ * happens inside the attention launch; for binary32 it is a separate launch first.
+ *   d_k, d_v   device [total][Hkv][D], the layer's rows of the appended chunk,
+ *              total and order as in the last append; 16-byte aligned
+ *   other arguments as for kvc_attn_prefill_chunk */
+int kvc_attn_prefill_chunk_kv(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v,
+                              const void* d_q, void* d_out, void* stream);
+
 /* Single-token decode GQA attention of one layer.  Sec. 3.1: after the unit's
  * first decision the model decodes, one token at a time, the transcription
  * segment (<|asr_start|>, up to 64 transcript tokens, <|asr_end|>) and, in SPEAK

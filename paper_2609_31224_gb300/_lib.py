@@ -26,7 +26,8 @@ STATUS = {0: "KVC_OK", -1: "KVC_EINVAL", -2: "KVC_ENOMEM", -3: "KVC_ECUDA", -4: 
 
 EXPORTED = ["kvc_query_sizes", "kvc_create", "kvc_destroy", "kvc_append_chunk",
             "kvc_append_kv_layer", "kvc_evict",
-            "kvc_attn_prefill_chunk", "kvc_attn_decode", "kvc_attn_decode_kv",
+            "kvc_attn_prefill_chunk", "kvc_attn_prefill_chunk_kv", "kvc_attn_decode",
+            "kvc_attn_decode_kv",
             "kvc_attn_decode_noalloc",
             "kvc_resident_size", "kvc_release",
             "kvc_export_state", "kvc_export_kv", "kvc_export_transcript", "kvc_device_status",
@@ -82,6 +83,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.kvc_attn_prefill_chunk.argtypes = [vp, ctypes.c_int, vp, vp, vp]
     lib.kvc_attn_decode.argtypes = [vp, ctypes.c_int, vp, vp, vp]
     lib.kvc_attn_decode_kv.argtypes = [vp, ctypes.c_int, vp, vp, vp, vp, vp]
+    lib.kvc_attn_prefill_chunk_kv.argtypes = [vp, ctypes.c_int, vp, vp, vp, vp, vp]
     lib.kvc_attn_decode_noalloc.argtypes = [vp, ctypes.c_int, vp, vp, vp]
     lib.kvc_resident_size.argtypes = [vp, ctypes.c_int, ctypes.POINTER(i64)]
     lib.kvc_release.argtypes = [vp, ctypes.c_int, p_i32, vp]
@@ -181,6 +183,12 @@ class KVCache:
 
     def attn_decode_raw(self, layer, q_ptr, out_ptr, stream) -> None:
         rc = self.lib.kvc_attn_decode(self.ctx, layer, q_ptr, out_ptr, stream)
+        if rc:
+            _check(rc)
+
+    def attn_prefill_kv_raw(self, layer, k_ptr, v_ptr, q_ptr, out_ptr, stream) -> None:
+        rc = self.lib.kvc_attn_prefill_chunk_kv(self.ctx, layer, k_ptr, v_ptr, q_ptr, out_ptr,
+                                                stream)
         if rc:
             _check(rc)
 

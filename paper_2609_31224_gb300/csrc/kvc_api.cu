@@ -521,6 +521,34 @@ int kvc_attn_prefill_chunk(kvc_ctx* ctx, int layer, const void* d_q, void* d_out
   return KVC_OK;
 }
 
+
+int kvc_attn_prefill_chunk_kv(kvc_ctx* ctx, int layer, const void* d_k, const void* d_v,
+                              const void* d_q, void* d_out, void* stream) {
+  g_err.clear();
+  int rc = check_attn(ctx, layer, d_q, d_out, true);
+  if (rc) return rc;
+  if (!d_k || !d_v) return fail(KVC_EINVAL, "d_k / d_v must be non-NULL");
+  if (!aligned16(d_k) || !aligned16(d_v)) return fail(KVC_EINVAL, "d_k / d_v must be 16-byte aligned");
+  if (ctx->last_max_t > PF_MAX_TOKENS)
+    return fail(KVC_EINVAL, "prefill chunks are limited to %d tokens per session", PF_MAX_TOKENS);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (ctx->d.esz == 2) {
+    // Launches after the append may start early: a stage holding chunk slots is
+    // copied only after its rows are written, and the previous launch writes
+    // another layer's rows only.
+    KVC_CUDA(launch_attn_prefill(ctx->d, layer, d_q, d_out, ctx->last_n_seq, ctx->last_max_t,
+                                 ctx->attn_since_append > 0, s, d_k, d_v));
+  } else {
+    // Binary32 (CUDA-core prefill): the rows first, then the attention, unoverlapped.
+    KVC_CUDA(launch_append_layers(ctx->d, ctx->last_total, layer, 1, d_k, d_v, s));
+    KVC_CUDA(launch_attn_prefill(ctx->d, layer, d_q, d_out, ctx->last_n_seq, ctx->last_max_t,
+                                 false, s));
+  }
+  ctx->layers_written |= 1ull << layer;
+  ++ctx->attn_since_append;
+  return KVC_OK;
+}
+
 int kvc_resident_size(kvc_ctx* ctx, int session, int64_t* h_out) {
   g_err.clear();
   if (!ctx || !h_out) return fail(KVC_EINVAL, "ctx / h_out is NULL");

@@ -265,7 +265,8 @@ int prefill_grid_ctas(const Dev& d) {
 }
 
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                                int max_t, bool pdl, cudaStream_t s) {
+                                int max_t, bool pdl, cudaStream_t s, const void* new_k,
+                                const void* new_v) {
   (void)n_seq;
   (void)max_t;
   if (d.esz == 2) {
@@ -275,8 +276,9 @@ cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* ou
     if (!gtc) gtc = pf_grid<0>(prefill_tc_kernel_ptr(), prefill_tc_threads(), prefill_tc_smem());
     // Each CTA of the stream-K split may write two partial slots.
     return launch_attn_prefill_tc(d, layer, lo, hi, q, out, std::min(gtc, d.max_pf_items / 2),
-                                  pdl, s);
+                                  pdl, s, new_k, new_v);
   }
+  if (new_k != nullptr) return cudaErrorInvalidValue;  // binary32: the API writes the rows first
   const float scale = LOG2E / sqrtf((float)d.head_dim);
   static thread_local int gf = 0;
   if (!gf) gf = pf_grid<0>(reinterpret_cast<const void*>(&attn_prefill_f32_kernel), F32_THREADS, 0);

@@ -25,6 +25,7 @@
 #include <cuda.h>
 
 #include "kvc_launch.cuh"
+#include "kvc_rope.cuh"
 
 namespace kvc {
 
@@ -173,6 +174,72 @@ __device__ inline uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo)
   return d;
 }
 
+// The per-layer write of the chunk rows of tokens [t0, t1) of a session (its call
+// row q_row0, positions from pos_first) for KV head `head`, by one warp: V rows
+// copied, or K rows rotated at their positions.  16-byte chunks, U per lane loaded
+// before any is stored.
+__device__ inline void write_chunk_rows(const Dev& d, int layer, const SeqInfo& si, int head,
+                                        bool is_v, const __nv_bfloat16* src, int t0, int t1,
+                                        int lane) {
+  constexpr int VEC = 8, HALF = D / 2, U = 4;
+  __nv_bfloat16* pool = reinterpret_cast<__nv_bfloat16*>(d.pool);
+  const int H = d.kv_heads;
+  const int per = is_v ? D / VEC : HALF / VEC;  // items per token
+  const int n = (t1 - t0) * per;
+  for (int base = lane; base < n; base += 32 * U) {
+    uint4 wa[U], wb[U];
+    float4 cs[U][VEC / 2];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int idx = base + 32 * u;
+      if (idx < n) {
+        const int t = t0 + idx / per, c = idx % per;
+        const __nv_bfloat16* row = src + ((size_t)(si.q_row0 + t) * H + head) * D + c * VEC;
+        wa[u] = *reinterpret_cast<const uint4*>(row);
+        if (!is_v) {
+          wb[u] = *reinterpret_cast<const uint4*>(row + HALF);
+          const float4* t4 =
+              reinterpret_cast<const float4*>(d.rope + (size_t)(si.pos_first + t) * HALF + c * VEC);
+#pragma unroll
+          for (int e = 0; e < VEC / 2; ++e) cs[u][e] = t4[e];
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int idx = base + 32 * u;
+      if (idx >= n) break;
+      const int t = t0 + idx / per, c = idx % per;
+      const int gs = d.tok_slot[si.q_row0 + t];
+      __nv_bfloat16* dst = pool + pool_offset_elems(d, gs / PS, layer, is_v ? 1 : 0, head, gs % PS) +
+                           c * VEC;
+      if (is_v) {
+        *reinterpret_cast<uint4*>(dst) = wa[u];
+      } else {
+        const __nv_bfloat16* xa = reinterpret_cast<const __nv_bfloat16*>(&wa[u]);
+        const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(&wb[u]);
+        uint4 ya, yb;
+        __nv_bfloat16* pa = reinterpret_cast<__nv_bfloat16*>(&ya);
+        __nv_bfloat16* pb = reinterpret_cast<__nv_bfloat16*>(&yb);
+#pragma unroll
+        for (int e = 0; e < VEC; ++e) {
+          const float4 tt = cs[u][e / 2];
+          float y1, y2;
+          rope_pair(__bfloat162float(xa[e]), __bfloat162float(xb[e]),
+                    (e & 1) ? make_float2(tt.z, tt.w) : make_float2(tt.x, tt.y), y1, y2);
+          pa[e] = __float2bfloat16_rn(y1);
+          pb[e] = __float2bfloat16_rn(y2);
+        }
+        *reinterpret_cast<uint4*>(dst) = ya;
+        *reinterpret_cast<uint4*>(dst + HALF) = yb;
+      }
+    }
+  }
+  // Order this lane's pool writes before the tensor copies the warp issues next.
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  __syncwarp();
+}
+
 // Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major, B K- or MN-major.
 __host__ __device__ constexpr uint32_t instr_desc(int n, int m, bool b_mn_major) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
@@ -190,10 +257,18 @@ __device__ inline float ex2(float x) {
   return y;
 }
 
+// FUSED (the per-layer order): the chunk's K (rotated at each token's position) and
+// V of this layer are not in the pool yet; new_k / new_v hold them ([total][Hkv][D],
+// the append's token order).  The producer warp that loads a stage holding chunk
+// slots of its (session, head) first writes those rows into the pool (the CTA
+// owning a (session, head, page) unit is the only reader of that unit in the
+// launch), then orders the writes before its tensor copy of the stage.
+template <bool FUSED>
 __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
     Dev d, int layer, const __grid_constant__ CUtensorMap map_lo,
     const __grid_constant__ CUtensorMap map_hi, const __nv_bfloat16* __restrict__ q,
-    __nv_bfloat16* __restrict__ out, float qk_scale) {
+    __nv_bfloat16* __restrict__ out, float qk_scale, const __nv_bfloat16* __restrict__ new_k,
+    const __nv_bfloat16* __restrict__ new_v) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -258,6 +333,8 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
     const int b_full = is_v ? B_V_FULL : B_K_FULL, b_empty = is_v ? B_V_EMPTY : B_K_EMPTY;
     uint32_t n = 0;  // stages produced
     bool stop = false;
+    bool waited = false;
+    (void)waited;
     for (int u = u_begin; u < u_end && !stop;) {
       const UnitSeg seg = unit_segment(d, u, u_end);
       u = seg.end;
@@ -287,6 +364,21 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
         int pages[4];
 #pragma unroll
         for (int pg = 0; pg < 4; ++pg) pages[pg] = __shfl_sync(FULL, pid, (b0 & 31) + pg);
+        if constexpr (FUSED) {
+          // Chunk tokens whose slots lie in this stage's blocks: their rows of this
+          // layer and head go into the pool before the stage is copied.
+          const int sl_first = si.live_head + si.n_live - si.t;
+          const int first_slot = (seg.u - seg.pair_start + b0 - si.n_hist_pages) * PS;
+          const int t0 = max(0, first_slot - sl_first);
+          const int t1 = min(si.t, first_slot + npg * PS - sl_first);
+          if (t0 < t1) {
+            if (!waited) {
+              pdl_wait();  // the rows may come from the kernel before this one
+              waited = true;
+            }
+            write_chunk_rows(d, layer, si, head, is_v, is_v ? new_v : new_k, t0, t1, lane);
+          }
+        }
         if (lane == 0) {
           mbar_arrive_expect_tx(&bars[b_full + st], npg * 2 * 2048);
           uint8_t* base = smem + OFF_KV + st * STAGE + (is_v ? 2 * KV_PANEL : 0);
@@ -642,18 +734,25 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
 }  // namespace
 
 const void* prefill_tc_kernel_ptr() {
-  return reinterpret_cast<const void*>(&attn_prefill_tc_kernel);
+  return reinterpret_cast<const void*>(&attn_prefill_tc_kernel<false>);
 }
 int prefill_tc_smem() { return TC_SMEM; }
 int prefill_tc_threads() { return THREADS; }
 
 cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,
                                    const CUtensorMap& hi, const void* q, void* out, int grid,
-                                   bool pdl, cudaStream_t s) {
+                                   bool pdl, cudaStream_t s, const void* new_k, const void* new_v) {
   const float scale = LOG2E / sqrtf((float)d.head_dim);
-  return launch_ex(&attn_prefill_tc_kernel, dim3(grid), dim3(THREADS), TC_SMEM, s, pdl, d, layer,
-                   lo, hi, static_cast<const __nv_bfloat16*>(q), static_cast<__nv_bfloat16*>(out),
-                   scale);
+  if (new_k != nullptr) {
+    static thread_local const cudaError_t attr = cudaFuncSetAttribute(
+        reinterpret_cast<const void*>(&attn_prefill_tc_kernel<true>),
+        cudaFuncAttributeMaxDynamicSharedMemorySize, TC_SMEM);
+    if (attr != cudaSuccess) return attr;
+  }
+  return launch_ex(new_k != nullptr ? &attn_prefill_tc_kernel<true> : &attn_prefill_tc_kernel<false>,
+                   dim3(grid), dim3(THREADS), TC_SMEM, s, pdl, d, layer, lo, hi,
+                   static_cast<const __nv_bfloat16*>(q), static_cast<__nv_bfloat16*>(out), scale,
+                   static_cast<const __nv_bfloat16*>(new_k), static_cast<const __nv_bfloat16*>(new_v));
 }
 
 }  // namespace kvc

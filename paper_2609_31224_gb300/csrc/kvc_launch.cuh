@@ -40,11 +40,22 @@ cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_o
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                bool pdl, cudaStream_t s, uint32_t epoch,
                                const void* new_k = nullptr, const void* new_v = nullptr);
+// Pair-split decode kernel (kvc_attn_decode_split.cu).  wide: the 16-warp shape
+// (one CTA per SM; tensor-core pages for bfloat16), else the 4-warp shape.
+int decode_split_slots(int esz, bool wide);          // resident CTAs in one wave
+bool decode_split_uses_tma(int esz, bool wide);      // needs the pool's tensor maps
+cudaError_t launch_attn_decode_split(const Dev& d, bool wide, int layer, const CUtensorMap& map_lo,
+                                     const CUtensorMap& map_hi, const void* q, void* out,
+                                     float scale, int k, uint32_t epoch, const void* new_k,
+                                     const void* new_v, int n_pairs, bool pdl, cudaStream_t s);
+// new_k / new_v (optional, bfloat16 only): the chunk's rows of this layer, written
+// into the pool by the launch itself (the per-layer order).
 cudaError_t launch_attn_prefill(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                                int max_t, bool pdl, cudaStream_t s);
+                                int max_t, bool pdl, cudaStream_t s, const void* new_k = nullptr,
+                                const void* new_v = nullptr);
 cudaError_t launch_attn_prefill_tc(const Dev& d, int layer, const CUtensorMap& lo,
                                    const CUtensorMap& hi, const void* q, void* out, int grid,
-                                   bool pdl, cudaStream_t s);
+                                   bool pdl, cudaStream_t s, const void* new_k, const void* new_v);
 const void* prefill_tc_kernel_ptr();
 // Two 2-D views of the bfloat16 pool as rows of 128 elements (columns 0-63 and
 // 64-127), 16-row boxes, 128-byte swizzle; cached per pool.  False if the driver

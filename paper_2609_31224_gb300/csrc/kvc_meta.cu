@@ -7,6 +7,7 @@
 // sessions' compacted-region pages are allocated before any live page is
 // freed).  This makes page tables a deterministic function of the calls.
 #include "kvc_launch.cuh"
+#include "kvc_rope.cuh"
 
 namespace kvc {
 
@@ -336,14 +337,6 @@ __global__ void __launch_bounds__(META_THREADS) append_plan_kernel(Dev d, Append
   }
 }
 
-// Rotate-half RoPE of one pair (x1, x2) = (k[j], k[j + D/2]) with (cos, sin) of
-// the position's angle for dim j, in binary32 on the binary32 table.  Every K
-// writer uses this one expression, so stored keys do not depend on the path.
-__device__ inline void rope_pair(float x1, float x2, float2 c, float& y1, float& y2) {
-  y1 = fmaf(x1, c.x, -x2 * c.y);
-  y2 = fmaf(x2, c.x, x1 * c.y);
-}
-
 // Append, part 2: K rotated at its position (rotate-half, binary32 math on
 // the binary32 table), V copied, both into the page slots of part 1.
 // grid = (tokens, layers); K/V input layout [L][total][Hkv][D].
@@ -491,84 +484,69 @@ __global__ void __launch_bounds__(META_THREADS) append_single_kernel(Dev d, Appe
   __syncthreads();
   // K rotated at the token's position and V, every layer and head: one 16-byte chunk
   // of the first half of a K row with its rotate-half partner per K item, one 16-byte
-  // chunk of V per V item; K/V input layout [L][n_seq][Hkv][D].  Each thread loads U
-  // items before it stores any, so their loads are in flight together.
-  constexpr int VEC = 16 / sizeof(T), U = 4;
+  // chunk of V per V item; K/V input layout [L][n_seq][Hkv][D].  Each thread loads
+  // its items of a pass before it stores any, so their loads are in flight together.
+  using CK = Chunk16<T>;
+  constexpr int VEC = CK::N, UK = sizeof(T) == 2 ? 1 : 2, UV = 4;
   const int D = d.head_dim, half = D / 2, H = d.kv_heads, L = d.layers;
   T* pool = reinterpret_cast<T*>(d.pool);
   const int kc = half / VEC, vc = D / VEC;
   const int n_k = n_seq * L * H * kc, n_v = n_seq * L * H * vc;
-  auto decompose = [&](int idx, int per, int& c, int& h, int& q, int& l) {
-    c = idx % per;
-    int r = idx / per;
-    h = r % H;
-    r /= H;
-    q = r % n_seq;
-    l = r / n_seq;
-  };
-  for (int base = i; base < n_k; base += U * META_THREADS) {
-    uint4 wa[U], wb[U];
-    float4 cs[U][VEC / 2];
+  for (int base = i; base < n_k; base += UK * META_THREADS) {
+    uint4 wa[UK], wb[UK];
+    float2 cs[UK][VEC];
+    int64_t dst_off[UK];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
+    for (int u = 0; u < UK; ++u) {
       const int idx = base + u * META_THREADS;
+      dst_off[u] = -1;
       if (idx < n_k) {
-        int c, h, q, l;
-        decompose(idx, kc, c, h, q, l);
+        const int c = idx % kc, r = idx / kc, h = r % H, q = (r / H) % n_seq, l = r / H / n_seq;
         const T* kin = k + (((size_t)l * n_seq + q) * H + h) * D + c * VEC;
         wa[u] = *reinterpret_cast<const uint4*>(kin);
         wb[u] = *reinterpret_cast<const uint4*>(kin + half);
-        const float4* t4 = reinterpret_cast<const float4*>(d.rope + (size_t)s_pos[q] * half + c * VEC);
+        const float2* t2 = d.rope + (size_t)s_pos[q] * half + c * VEC;
 #pragma unroll
-        for (int e = 0; e < VEC / 2; ++e) cs[u][e] = t4[e];
+        for (int e = 0; e < VEC; ++e) cs[u][e] = t2[e];
+        const int gs = s_gs[q];
+        dst_off[u] = (int64_t)(pool_offset_elems(d, gs / PS, l, 0, h, gs % PS) + c * VEC);
       }
     }
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int idx = base + u * META_THREADS;
-      if (idx >= n_k) break;
-      int c, h, q, l;
-      decompose(idx, kc, c, h, q, l);
-      const T* xa = reinterpret_cast<const T*>(&wa[u]);
-      const T* xb = reinterpret_cast<const T*>(&wb[u]);
-      uint4 ya, yb;
-      T* pa = reinterpret_cast<T*>(&ya);
-      T* pb = reinterpret_cast<T*>(&yb);
+    for (int u = 0; u < UK; ++u) {
+      if (dst_off[u] < 0) break;
+      float xa[VEC], xb[VEC], ya[VEC], yb[VEC];
+      CK::unpack(wa[u], xa);
+      CK::unpack(wb[u], xb);
 #pragma unroll
       for (int e = 0; e < VEC; ++e) {
-        const float4 t = cs[u][e / 2];
-        const float2 ce = (e & 1) ? make_float2(t.z, t.w) : make_float2(t.x, t.y);
         float y1, y2;
-        rope_pair(to_float<T>(xa[e]), to_float<T>(xb[e]), ce, y1, y2);
-        pa[e] = from_float<T>(y1);
-        pb[e] = from_float<T>(y2);
+        rope_pair(xa[e], xb[e], cs[u][e], y1, y2);
+        ya[e] = y1;
+        yb[e] = y2;
       }
-      const int gs = s_gs[q];
-      T* dst = pool + pool_offset_elems(d, gs / PS, l, 0, h, gs % PS) + c * VEC;
-      *reinterpret_cast<uint4*>(dst) = ya;
-      *reinterpret_cast<uint4*>(dst + half) = yb;
+      *reinterpret_cast<uint4*>(pool + dst_off[u]) = CK::pack(ya);
+      *reinterpret_cast<uint4*>(pool + dst_off[u] + half) = CK::pack(yb);
     }
   }
-  for (int base = i; base < n_v; base += U * META_THREADS) {
-    uint4 x[U];
+  for (int base = i; base < n_v; base += UV * META_THREADS) {
+    uint4 x[UV];
+    int64_t dst_off[UV];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
+    for (int u = 0; u < UV; ++u) {
       const int idx = base + u * META_THREADS;
+      dst_off[u] = -1;
       if (idx < n_v) {
-        int c, h, q, l;
-        decompose(idx, vc, c, h, q, l);
+        const int c = idx % vc, r = idx / vc, h = r % H, q = (r / H) % n_seq, l = r / H / n_seq;
         x[u] = *reinterpret_cast<const uint4*>(v + (((size_t)l * n_seq + q) * H + h) * D + c * VEC);
+        const int gs = s_gs[q];
+        dst_off[u] = (int64_t)(pool_offset_elems(d, gs / PS, l, 1, h, gs % PS) + c * VEC);
       }
     }
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int idx = base + u * META_THREADS;
-      if (idx >= n_v) break;
-      int c, h, q, l;
-      decompose(idx, vc, c, h, q, l);
-      const int gs = s_gs[q];
-      *reinterpret_cast<uint4*>(pool + pool_offset_elems(d, gs / PS, l, 1, h, gs % PS) + c * VEC) =
-          x[u];
+    for (int u = 0; u < UV; ++u) {
+      if (dst_off[u] < 0) break;
+      *reinterpret_cast<uint4*>(pool + dst_off[u]) = x[u];
     }
   }
 }

@@ -178,7 +178,9 @@ class Driver:
         """Append + (optionally) every layer's attention. Returns kernels launched.
 
         per_layer: the model's order; the append carries no K/V and each layer's K/V
-        are written just before that layer's attention."""
+        are written by that layer's attention call (kvc_attn_decode_kv,
+        kvc_attn_prefill_chunk_kv), or, for calls without attention, just before it
+        would run (kvc_append_kv_layer)."""
         cache = self.cache
         _, s_p, _, c_p, t_ptr, k_ptr, v_ptr, q_ptrs, o_ptr = c.raw
         stream = self.stream
@@ -192,10 +194,12 @@ class Driver:
         kv_stride = c.k.stride(0) * c.k.element_size()
         for layer in range(self.w.layers):
             kl, vl = k_ptr + layer * kv_stride, v_ptr + layer * kv_stride
-            if per_layer and do_attn and c.kind == "decode":
-                # The layer's K/V write fused into its decode launch.
-                cache.attn_decode_kv_raw(layer, kl, vl, q_ptrs[layer], o_ptr, stream)
-                launches += 1
+            if per_layer and do_attn:
+                # The layer's K/V write fused into its attention call.
+                fused = (cache.attn_decode_kv_raw if c.kind == "decode"
+                         else cache.attn_prefill_kv_raw)
+                fused(layer, kl, vl, q_ptrs[layer], o_ptr, stream)
+                launches += 1 if (c.kind == "decode" or self.w.dtype == "bf16") else 2
                 if on_attention is not None:
                     on_attention(c, layer)
                 continue

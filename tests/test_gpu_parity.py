@@ -170,6 +170,20 @@ def test_per_layer_append(dtype):
     assert ls.n_compared > 0
 
 
+def test_per_layer_append_batch64_prefill():
+    """The model's order at the 64-session prefill size: every prefill call (64 sessions x
+    17 positions) writes its layer's rows inside the tensor-core attention launch
+    (kvc_attn_prefill_chunk_kv) and every decode call inside the decode launch; all
+    outputs of sampled layers compared with the oracle, every evict bit-exact."""
+    w = S.SINGLE_BF16.with_(layers=4, n_sessions=64, budget=300, window=2, seed=41,
+                            offset_max=2, turn_period=9, turn_jitter=1)
+    ls, _ = _lockstep(w, n_units=18)
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(attn_pred=lambda st, kind, i, layer: layer in (0, 3) and
+                    (kind == "prefill" or st % 4 == 0), per_layer=True)
+    assert ls.n_compared > 64 * 2 * 10
+
+
 def test_fused_layer_write_stores_the_same_bytes():
     """Whole-chunk appends and the per-layer order (separate writes for prefill chunks,
     writes fused into the decode launches) leave bit-identical K/V in every layer."""
