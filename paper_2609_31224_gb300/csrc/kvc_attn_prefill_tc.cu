@@ -70,7 +70,10 @@ enum {
   B_O = B_P_EMPTY + 2,
   B_Q = B_O + 2,                         // one phase per segment (query tile ready)
   B_FINAL = B_Q + 1,                     // every MMA of the CTA complete (both issuers)
-  N_BARS = B_FINAL + 1
+  // Fused layer write: one phase per segment holding chunk slots, completed when the
+  // softmax warps have written those rows into the pool.
+  B_ROWS = B_FINAL + 1,
+  N_BARS = B_ROWS + 1
 };
 constexpr int OFF_TMEM_ADDR = OFF_BAR + N_BARS * 8;
 constexpr int TC_SMEM = OFF_TMEM_ADDR + 16 + 1024;  // + alignment slack
@@ -175,69 +178,52 @@ __device__ inline uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo)
 }
 
 // The per-layer write of the chunk rows of tokens [t0, t1) of a session (its call
-// row q_row0, positions from pos_first) for KV head `head`, by one warp: V rows
-// copied, or K rows rotated at their positions.  16-byte chunks, U per lane loaded
-// before any is stored.
+// row q_row0, positions from pos_first) for KV head `head`, by the 128 softmax
+// threads (thread index ts): V rows copied, K rows rotated at their positions, in
+// 16-byte chunks, every load of an item issued before its stores.  Each thread then
+// orders its writes before later tensor copies (async proxy).
 __device__ inline void write_chunk_rows(const Dev& d, int layer, const SeqInfo& si, int head,
-                                        bool is_v, const __nv_bfloat16* src, int t0, int t1,
-                                        int lane) {
-  constexpr int VEC = 8, HALF = D / 2, U = 4;
+                                        const __nv_bfloat16* new_k, const __nv_bfloat16* new_v,
+                                        int t0, int t1, int ts) {
+  // Item (token, c): 16-byte chunk c of the first half of the K row with its
+  // rotate-half partner, and chunks c and c + 8 of the V row.
+  constexpr int VEC = 8, HALF = D / 2, KC = HALF / VEC;
   __nv_bfloat16* pool = reinterpret_cast<__nv_bfloat16*>(d.pool);
   const int H = d.kv_heads;
-  const int per = is_v ? D / VEC : HALF / VEC;  // items per token
-  const int n = (t1 - t0) * per;
-  for (int base = lane; base < n; base += 32 * U) {
-    uint4 wa[U], wb[U];
-    float4 cs[U][VEC / 2];
+  const int n = (t1 - t0) * KC;
+  for (int idx = ts; idx < n; idx += 128) {
+    const int t = t0 + idx / KC, c = idx % KC;
+    const size_t in_row = ((size_t)(si.q_row0 + t) * H + head) * D + c * VEC;
+    const uint4 ka = *reinterpret_cast<const uint4*>(new_k + in_row);
+    const uint4 kb = *reinterpret_cast<const uint4*>(new_k + in_row + HALF);
+    const uint4 va = *reinterpret_cast<const uint4*>(new_v + in_row);
+    const uint4 vb = *reinterpret_cast<const uint4*>(new_v + in_row + HALF);
+    const float2* t2 = d.rope + (size_t)(si.pos_first + t) * HALF + c * VEC;
+    float2 cs[VEC];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int idx = base + 32 * u;
-      if (idx < n) {
-        const int t = t0 + idx / per, c = idx % per;
-        const __nv_bfloat16* row = src + ((size_t)(si.q_row0 + t) * H + head) * D + c * VEC;
-        wa[u] = *reinterpret_cast<const uint4*>(row);
-        if (!is_v) {
-          wb[u] = *reinterpret_cast<const uint4*>(row + HALF);
-          const float4* t4 =
-              reinterpret_cast<const float4*>(d.rope + (size_t)(si.pos_first + t) * HALF + c * VEC);
+    for (int e = 0; e < VEC; ++e) cs[e] = t2[e];
+    const int gs = d.tok_slot[si.q_row0 + t];
+    float xa[VEC], xb[VEC], ya[VEC], yb[VEC];
+    Chunk16<__nv_bfloat16>::unpack(ka, xa);
+    Chunk16<__nv_bfloat16>::unpack(kb, xb);
 #pragma unroll
-          for (int e = 0; e < VEC / 2; ++e) cs[u][e] = t4[e];
-        }
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int idx = base + 32 * u;
-      if (idx >= n) break;
-      const int t = t0 + idx / per, c = idx % per;
-      const int gs = d.tok_slot[si.q_row0 + t];
-      __nv_bfloat16* dst = pool + pool_offset_elems(d, gs / PS, layer, is_v ? 1 : 0, head, gs % PS) +
-                           c * VEC;
-      if (is_v) {
-        *reinterpret_cast<uint4*>(dst) = wa[u];
-      } else {
-        const __nv_bfloat16* xa = reinterpret_cast<const __nv_bfloat16*>(&wa[u]);
-        const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(&wb[u]);
-        uint4 ya, yb;
-        __nv_bfloat16* pa = reinterpret_cast<__nv_bfloat16*>(&ya);
-        __nv_bfloat16* pb = reinterpret_cast<__nv_bfloat16*>(&yb);
-#pragma unroll
-        for (int e = 0; e < VEC; ++e) {
-          const float4 tt = cs[u][e / 2];
-          float y1, y2;
-          rope_pair(__bfloat162float(xa[e]), __bfloat162float(xb[e]),
-                    (e & 1) ? make_float2(tt.z, tt.w) : make_float2(tt.x, tt.y), y1, y2);
-          pa[e] = __float2bfloat16_rn(y1);
-          pb[e] = __float2bfloat16_rn(y2);
-        }
-        *reinterpret_cast<uint4*>(dst) = ya;
-        *reinterpret_cast<uint4*>(dst + HALF) = yb;
-      }
-    }
+    for (int e = 0; e < VEC; ++e) rope_pair(xa[e], xb[e], cs[e], ya[e], yb[e]);
+    __nv_bfloat16* kd = pool + pool_offset_elems(d, gs / PS, layer, 0, head, gs % PS) + c * VEC;
+    __nv_bfloat16* vd = pool + pool_offset_elems(d, gs / PS, layer, 1, head, gs % PS) + c * VEC;
+    *reinterpret_cast<uint4*>(kd) = Chunk16<__nv_bfloat16>::pack(ya);
+    *reinterpret_cast<uint4*>(kd + HALF) = Chunk16<__nv_bfloat16>::pack(yb);
+    *reinterpret_cast<uint4*>(vd) = va;
+    *reinterpret_cast<uint4*>(vd + HALF) = vb;
   }
-  // Order this lane's pool writes before the tensor copies the warp issues next.
   asm volatile("fence.proxy.async.global;" ::: "memory");
-  __syncwarp();
+}
+
+// Chunk tokens [t0, t1) of a session whose slots lie in its blocks [b_lo, b_hi).
+__device__ inline void chunk_tokens_in(const SeqInfo& si, int b_lo, int b_hi, int& t0, int& t1) {
+  const int sl_first = si.live_head + si.n_live - si.t;  // live slot of the first token
+  const int lo = (b_lo - si.n_hist_pages) * PS, hi = (b_hi - si.n_hist_pages) * PS;
+  t0 = max(0, lo - sl_first);
+  t1 = min(si.t, hi - sl_first);
 }
 
 // Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major, B K- or MN-major.
@@ -295,6 +281,7 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
     mbar_init(&bars[B_O + 1], 1);
     mbar_init(&bars[B_Q], 4);
     mbar_init(&bars[B_FINAL], 2);
+    mbar_init(&bars[B_ROWS], 4);
     fence_mbar_init();
     s_abort = 0;
   }
@@ -333,8 +320,8 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
     const int b_full = is_v ? B_V_FULL : B_K_FULL, b_empty = is_v ? B_V_EMPTY : B_K_EMPTY;
     uint32_t n = 0;  // stages produced
     bool stop = false;
-    bool waited = false;
-    (void)waited;
+    uint32_t rows_seen = 0;  // segments holding chunk slots, before this one
+    (void)rows_seen;
     for (int u = u_begin; u < u_end && !stop;) {
       const UnitSeg seg = unit_segment(d, u, u_end);
       u = seg.end;
@@ -345,6 +332,20 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       const int blk0 = seg.blk_begin(), nblk = seg.end - seg.u;
       const int n_st = (nblk + 3) / 4;
       int pid = 0;
+      if (is_v) {
+        // The segment's query rows (T tokens x G heads, 1 KiB per token) and rotary
+        // rows (512 B per token) into L2 ahead of the softmax warps, which read them
+        // when the segment starts.  A prefetch changes nothing that a later load
+        // observes, so it may run before the previous kernel has finished.
+        const char* qb = reinterpret_cast<const char*>(
+            q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G) * D);
+        const char* rb = reinterpret_cast<const char*>(d.rope + (size_t)si.pos_first * (D / 2));
+        const size_t qstride = (size_t)d.q_heads * D * sizeof(__nv_bfloat16);
+        for (int x = lane; x < si.t * 12; x += 32) {
+          const int tt = x / 12, line = x % 12;
+          prefetch_l2(line < 8 ? qb + tt * qstride + line * 128 : rb + (size_t)tt * 512 + (line - 8) * 128);
+        }
+      }
       for (int k = 0; k < n_st; ++k, ++n) {
         const int b0 = 4 * k;
         if ((b0 & 31) == 0) {
@@ -365,18 +366,18 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
 #pragma unroll
         for (int pg = 0; pg < 4; ++pg) pages[pg] = __shfl_sync(FULL, pid, (b0 & 31) + pg);
         if constexpr (FUSED) {
-          // Chunk tokens whose slots lie in this stage's blocks: their rows of this
-          // layer and head go into the pool before the stage is copied.
-          const int sl_first = si.live_head + si.n_live - si.t;
-          const int first_slot = (seg.u - seg.pair_start + b0 - si.n_hist_pages) * PS;
-          const int t0 = max(0, first_slot - sl_first);
-          const int t1 = min(si.t, first_slot + npg * PS - sl_first);
+          // A stage holding chunk slots is copied only once the softmax warps have
+          // written the segment's rows (they do so when the segment starts).
+          int t0, t1;
+          chunk_tokens_in(si, blk0 + b0, blk0 + b0 + npg, t0, t1);
           if (t0 < t1) {
-            if (!waited) {
-              pdl_wait();  // the rows may come from the kernel before this one
-              waited = true;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(d, &bars[B_ROWS], rows_seen & 1);
+            if (!__shfl_sync(FULL, ok, 0)) {
+              if (lane == 0) s_abort = 1;
+              stop = true;
+              break;
             }
-            write_chunk_rows(d, layer, si, head, is_v, is_v ? new_v : new_k, t0, t1, lane);
           }
         }
         if (lane == 0) {
@@ -389,6 +390,11 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
             tma_load_2d(base + KV_PANEL + pg * 2048, &map_hi, 0, row, &bars[b_full + st]);
           }
         }
+      }
+      if constexpr (FUSED) {
+        int t0, t1;
+        chunk_tokens_in(si, blk0, blk0 + nblk, t0, t1);
+        if (t0 < t1) ++rows_seen;
       }
       stop = stop || __any_sync(FULL, s_abort != 0);
     }
@@ -539,6 +545,15 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars[B_Q]);
+      if constexpr (FUSED) {
+        int t0, t1;
+        chunk_tokens_in(si, blk0, blk0 + nblk, t0, t1);
+        if (t0 < t1) {
+          if (!dead) write_chunk_rows(d, layer, si, head, new_k, new_v, t0, t1, r);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars[B_ROWS]);
+        }
+      }
 
       // Blocks that may need a mask: the partly filled last history page, the
       // first live page when it starts mid-page, and every block from the one

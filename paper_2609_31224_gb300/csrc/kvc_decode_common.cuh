@@ -245,20 +245,37 @@ __device__ void patch_new_row(const Dev& d, int layer, const SeqInfo& si, int he
     else
       return slot * C::ROW_BYTES + j * C::ESZ;
   };
-  for (int j = lane; j < HALF; j += 32) {
-    const float x1 = to_float<T>(kin[j]), x2 = to_float<T>(kin[j + HALF]);
-    const float2 c = cs[j];
-    const T y1 = from_float<T>(fmaf(x1, c.x, -x2 * c.y));
-    const T y2 = from_float<T>(fmaf(x2, c.x, x1 * c.y));
+  // Every load of the row is issued before any store (one round trip): lane owns the
+  // rotate-half pairs (j, j + D/2) for j = lane + 32 i and the V elements lane + 32 i.
+  constexpr int KP = HALF / 32, VP = D / 32;
+  static_assert(HALF % 32 == 0, "whole pairs per lane");
+  float x1[KP], x2[KP];
+  float2 c[KP];
+  T vv[VP];
+#pragma unroll
+  for (int i = 0; i < KP; ++i) {
+    const int j = lane + 32 * i;
+    x1[i] = to_float<T>(kin[j]);
+    x2[i] = to_float<T>(kin[j + HALF]);
+    c[i] = cs[j];
+  }
+#pragma unroll
+  for (int i = 0; i < VP; ++i) vv[i] = vin[lane + 32 * i];
+#pragma unroll
+  for (int i = 0; i < KP; ++i) {
+    const int j = lane + 32 * i;
+    const T y1 = from_float<T>(fmaf(x1[i], c[i].x, -x2[i] * c[i].y));
+    const T y2 = from_float<T>(fmaf(x2[i], c[i].x, x1[i] * c[i].y));
     *reinterpret_cast<T*>(kt + at(j)) = y1;
     *reinterpret_cast<T*>(kt + at(j + HALF)) = y2;
     kp[j] = y1;
     kp[j + HALF] = y2;
   }
-  for (int j = lane; j < D; j += 32) {
-    const T x = vin[j];
-    *reinterpret_cast<T*>(kt + C::TILE + at(j)) = x;
-    vp[j] = x;
+#pragma unroll
+  for (int i = 0; i < VP; ++i) {
+    const int j = lane + 32 * i;
+    *reinterpret_cast<T*>(kt + C::TILE + at(j)) = vv[i];
+    vp[j] = vv[i];
   }
   __syncwarp();
 }
