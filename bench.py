@@ -38,13 +38,14 @@ UNIT = "audio-s/s"
 
 # DRAM bytes per algorithmic byte of the roofline kernel (reads + writes), from one
 # ncu capture of the stream-K kernel on the 24-session, two-layer reduced case:
-# 410.69 MB of traffic (406.84 MB read, 3.85 MB written) for a 403.97 MB launch.  Valid only while the decode sources
-# hash to the version it was taken on; the roofline's traffic is null otherwise.
-DECODE_TRAFFIC_RATIO = 410.69 / 403.97
+# 409.79 MB of traffic (406.83 MB read, 2.97 MB written) for a 403.97 MB launch.  Valid only
+# while the decode sources hash to the version it was taken on; the roofline's traffic is
+# null otherwise.
+DECODE_TRAFFIC_RATIO = 409.79 / 403.97
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
                           "paper_2609_31224_gb300/csrc/kvc_decode_common.cuh",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "827208e31cdde3946b24310eec0fba47957f0a4139e83994ba0fcce1a6e5529b"
+DECODE_TRAFFIC_SHA256 = "463ff4e942d77aeda9e12db0da7a1ddc1b0243ecdbefce712a590c92d790e1d4"
 
 
 def decode_traffic(alg_bytes_per_launch):
@@ -386,6 +387,9 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
         host.append(hs)
         dev.append(ds)
     res_host = torch.empty(w.n_sessions, dtype=torch.int64).pin_memory()
+    # One resident-count buffer per step: a step's evict never overwrites counts that
+    # the result stream has not copied yet.
+    res_dev = torch.zeros((n_steps, w.n_sessions), dtype=torch.int64, device="cuda")
     out_host = [[torch.empty(c.out.shape, dtype=c.out.dtype).pin_memory() if c.out is not None
                  else None for c in st.calls] for st in steps]
     h2d = sum(t.numel() * t.element_size() for hs in host[0] for t in hs.values())
@@ -396,8 +400,11 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
         torch.distributed.barrier()
     # Inputs move on a copy stream, one step ahead of the compute: step i+1's copies are
     # enqueued just before step i's launches, and each step's compute waits only for its
-    # own inputs, so transfers overlap the previous step's compute.
+    # own inputs, so transfers overlap the previous step's compute.  Results come back on
+    # a third stream, each after an event behind the call that wrote it, so the compute
+    # stream never queues behind a copy.
     copy_stream = torch.cuda.Stream()
+    d2h_stream = torch.cuda.Stream()
     copy_start = [torch.cuda.Event(enable_timing=True) for _ in steps]
     comp = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
             for _ in steps]
@@ -406,6 +413,7 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     copy_stream.wait_stream(stream)
+    d2h_stream.wait_stream(stream)
     h2d_total, d2h_total = 0, 0
 
     def enqueue_copies(si):
@@ -427,13 +435,18 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
         for ci, c in enumerate(st.calls):
             drv.run_call(c, per_layer=per_layer)
             if c.out is not None:
-                out_host[si][ci].copy_(c.out, non_blocking=True)
+                d2h_stream.wait_stream(stream)
+                with torch.cuda.stream(d2h_stream):
+                    out_host[si][ci].copy_(c.out, non_blocking=True)
                 d2h_total += c.out.numel() * c.out.element_size()
-        drv.cache.evict(st.evict_sessions, drv.resident_out)
+        drv.cache.evict(st.evict_sessions, res_dev[si])
         n = len(st.evict_sessions)
-        res_host[:n].copy_(drv.resident_out[:n], non_blocking=True)
+        d2h_stream.wait_stream(stream)
+        with torch.cuda.stream(d2h_stream):
+            res_host[:n].copy_(res_dev[si, :n], non_blocking=True)
         d2h_total += n * 8
         comp[si][1].record(stream)
+    stream.wait_stream(d2h_stream)
     e1.record(stream)
     submit = time.perf_counter() - t0
     torch.cuda.synchronize()

@@ -17,6 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkvc.so")
 SOURCES = ["kvc_api.cu", "kvc_meta.cu", "kvc_attn_decode.cu", "kvc_attn_decode_split.cu",
+           "kvc_decode_dispatch.cu",
            "kvc_attn_prefill.cu", "kvc_attn_prefill_tc.cu", "kvc_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

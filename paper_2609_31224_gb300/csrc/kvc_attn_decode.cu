@@ -22,10 +22,9 @@
 // whose tag is not yet current.  Launches captured into a graph (where a replay
 // would repeat the tag) use the acquire-release arrival.
 //
-// This file holds the stream-K kernel and the dispatch between the tiers; the
-// pair-split kernel is in kvc_attn_decode_split.cu.
-#include <cstring>
-
+// This file holds the stream-K kernel; the pair-split kernel is in
+// kvc_attn_decode_split.cu and the dispatch between the tiers in
+// kvc_decode_dispatch.cu.
 #include "kvc_decode_common.cuh"
 
 namespace kvc {
@@ -154,56 +153,31 @@ int stream_k_grid(const Dev& d) {
   return min(d.dec_slots / 2, max(1, per_sm) * sms);
 }
 
-// Minimum (session, kv head, page) units per CTA of the stream-K split.
-constexpr int DEC_MIN_UNITS = 12;
-// The pair-split kernel takes calls whose pairs each get at least this many CTAs
-// in one wave: with 16-warp CTAs (one per SM) first, else with stream-K's 4-warp
-// CTAs (three per SM).  Only the 16-warp shape uses tagged partial states: with
-// 4-warp CTAs the fenced arrival measured faster.
-constexpr int SPLIT_MIN_K = 2, SPLIT4_MIN_K = 3;
-
-template <typename T, int D>
-cudaError_t launch_decode(const Dev& d, int layer, const void* q, void* out, int n_seq, bool pdl,
-                          cudaStream_t s, uint32_t epoch, const void* new_k, const void* new_v) {
-  static thread_local const int grid = stream_k_grid<T, D>(d);
-  static thread_local const int slots = decode_split_slots(sizeof(T), true);
-  static thread_local const int slots4 = decode_split_slots(sizeof(T), false);
-  const float scale = LOG2E / sqrtf((float)D);
-  const int n_pairs = n_seq * d.kv_heads;
-  const int k = n_pairs * SPLIT_MIN_K <= slots ? min(MAX_PARTS, slots / n_pairs) : 0;
-  const int k4 = k == 0 && n_pairs * SPLIT4_MIN_K <= slots4 ? min(MAX_PARTS, slots4 / n_pairs) : 0;
-  // Tensor maps of the pool for the tensor-core page loop (bfloat16).
-  CUtensorMap map_lo, map_hi;
-  memset(&map_lo, 0, sizeof(map_lo));
-  memset(&map_hi, 0, sizeof(map_hi));
-  if (((k > 0 && decode_split_uses_tma(sizeof(T), true)) ||
-       (k4 > 0 && decode_split_uses_tma(sizeof(T), false))) &&
-      !pool_tensor_maps(d, &map_lo, &map_hi))
-    return cudaErrorInvalidValue;
-  if (k > 0)
-    return launch_attn_decode_split(d, true, layer, map_lo, map_hi, q, out, scale, k,
-                                    n_pairs * k <= d.dec_tag_slots ? epoch : 0u, new_k, new_v,
-                                    n_pairs, pdl, s);
-  if (k4 > 0)
-    return launch_attn_decode_split(d, false, layer, map_lo, map_hi, q, out, scale, k4, 0u, new_k,
-                                    new_v, n_pairs, pdl, s);
-  const T* nk = static_cast<const T*>(new_k);
-  const T* nv = static_cast<const T*>(new_v);
-  return launch_ex(nk ? &attn_decode_kernel<T, D, true> : &attn_decode_kernel<T, D, false>,
-                   dim3(grid), dim3(SkCfg<T, D>::THREADS), SkCfg<T, D>::SMEM, s, pdl, d, layer,
-                   map_lo, map_hi, static_cast<const T*>(q), static_cast<T*>(out), scale,
-                   DEC_MIN_UNITS, nk, nv);
-}
-
 }  // namespace
 
-cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
-                               bool pdl, cudaStream_t s, uint32_t epoch, const void* new_k,
-                               const void* new_v) {
-  if (d.esz == 2)
-    return launch_decode<__nv_bfloat16, 128>(d, layer, q, out, n_seq, pdl, s, epoch, new_k,
-                                             new_v);
-  return launch_decode<float, 64>(d, layer, q, out, n_seq, pdl, s, epoch, new_k, new_v);
+int decode_stream_k_grid(const Dev& d) {
+  return d.esz == 2 ? stream_k_grid<__nv_bfloat16, 128>(d) : stream_k_grid<float, 64>(d);
+}
+
+cudaError_t launch_attn_decode_streamk(const Dev& d, int layer, const CUtensorMap& map_lo,
+                                       const CUtensorMap& map_hi, const void* q, void* out,
+                                       float scale, int grid, int min_units, const void* new_k,
+                                       const void* new_v, bool pdl, cudaStream_t s) {
+  if (d.esz == 2) {
+    using T = __nv_bfloat16;
+    const T* nk = static_cast<const T*>(new_k);
+    const T* nv = static_cast<const T*>(new_v);
+    return launch_ex(nk ? &attn_decode_kernel<T, 128, true> : &attn_decode_kernel<T, 128, false>,
+                     dim3(grid), dim3(SkCfg<T, 128>::THREADS), SkCfg<T, 128>::SMEM, s, pdl, d,
+                     layer, map_lo, map_hi, static_cast<const T*>(q), static_cast<T*>(out), scale,
+                     min_units, nk, nv);
+  }
+  const float* nk = static_cast<const float*>(new_k);
+  const float* nv = static_cast<const float*>(new_v);
+  return launch_ex(nk ? &attn_decode_kernel<float, 64, true> : &attn_decode_kernel<float, 64, false>,
+                   dim3(grid), dim3(SkCfg<float, 64>::THREADS), SkCfg<float, 64>::SMEM, s, pdl, d,
+                   layer, map_lo, map_hi, static_cast<const float*>(q), static_cast<float*>(out),
+                   scale, min_units, nk, nv);
 }
 
 }  // namespace kvc

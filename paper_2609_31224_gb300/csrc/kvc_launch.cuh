@@ -40,6 +40,13 @@ cudaError_t launch_transcript(const Dev& d, int session, int cap, int32_t* pos_o
 cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out, int n_seq,
                                bool pdl, cudaStream_t s, uint32_t epoch,
                                const void* new_k = nullptr, const void* new_v = nullptr);
+// Stream-K decode kernel (kvc_attn_decode.cu): its grid (resident CTAs, capped by
+// the partial slots) and its launch.
+int decode_stream_k_grid(const Dev& d);
+cudaError_t launch_attn_decode_streamk(const Dev& d, int layer, const CUtensorMap& map_lo,
+                                       const CUtensorMap& map_hi, const void* q, void* out,
+                                       float scale, int grid, int min_units, const void* new_k,
+                                       const void* new_v, bool pdl, cudaStream_t s);
 // Pair-split decode kernel (kvc_attn_decode_split.cu).  wide: the 16-warp shape
 // (one CTA per SM; tensor-core pages for bfloat16), else the 4-warp shape.
 int decode_split_slots(int esz, bool wide);          // resident CTAs in one wave
