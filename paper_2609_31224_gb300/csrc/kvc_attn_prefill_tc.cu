@@ -693,47 +693,110 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
           s_last = arrive_acq_rel(&d.pf_count[seg.seq * H + head], nch);
         asm volatile("bar.sync 1, 128;" ::: "memory");
         if (s_last) {
-          if (live) {
-            const int first_slot = us.slot_of(cf, cf, seg.pair_start);
-            auto prow = [&](int ch) {
-              return (size_t)(ch ? 2 * (cf + ch) : first_slot) * (PF_MAX_TOKENS * G) + r;
-            };
-            float Mx = -INFINITY;
-            for (int ch = 0; ch < nch; ++ch) Mx = fmaxf(Mx, __ldcg(&d.pf_part_ml[prow(ch)]).x);
-            float Ls = 0.f;
-            for (int ch = 0; ch < nch; ++ch) {
-              const float2 ml = __ldcg(&d.pf_part_ml[prow(ch)]);
-              Ls += ml.y * exp2_safe(ml.x, Mx);
-            }
-            const float invL = 1.f / Ls;
-            __nv_bfloat16* orow =
-                out + ((size_t)(si.q_row0 + t) * d.q_heads + head * G + g) * D;
-            for (int c = 0; c < D / 32; ++c) {
-              float acc[32];
+          // The merge runs in tensor memory: this CTA's own part is still in the O
+          // columns (the next segment's first P V overwrites them only after this),
+          // and each other part's row is loaded whole, all its words at once, and
+          // added there.  The first other part's row is loaded together with every
+          // part's (max, sum), so a pair of two parts costs one round trip.  Every
+          // lane takes part in the tensor-memory accesses; rows that are padding (or
+          // of a warp whose wait gave up) weigh 0 and write nothing.
+          const int first_slot = us.slot_of(cf, cf, seg.pair_start);
+          const int own = cta - cf;
+          auto prow = [&](int ch) {
+            return (size_t)(ch ? 2 * (cf + ch) : first_slot) * (PF_MAX_TOKENS * G) + r;
+          };
+          auto load_row = [&](int ch, float4 (&v)[D / 4]) {
+            const float4* src = reinterpret_cast<const float4*>(d.pf_part_o + prow(ch) * D);
 #pragma unroll
-              for (int i = 0; i < 32; ++i) acc[i] = 0.f;
-              for (int ch = 0; ch < nch; ++ch) {
-                const size_t row = prow(ch);
-                const float sc2 = exp2_safe(__ldcg(&d.pf_part_ml[row]).x, Mx) * invL;
-                const float4* src =
-                    reinterpret_cast<const float4*>(d.pf_part_o + row * D + c * 32);
+            for (int i = 0; i < D / 4; ++i)
+              v[i] = write ? __ldcg(src + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+          };
+          const int f0 = own == 0 ? 1 : 0;  // first other part
+          float4 v[D / 4];
+          load_row(f0, v);
+          constexpr int MB = 8;
+          float2 ml[MB];
+          auto load_ml = [&](int c0) {
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                  const float4 v = __ldcg(src + i);
-                  acc[4 * i] += v.x * sc2;
-                  acc[4 * i + 1] += v.y * sc2;
-                  acc[4 * i + 2] += v.z * sc2;
-                  acc[4 * i + 3] += v.w * sc2;
-                }
-              }
+            for (int i = 0; i < MB; ++i)
+              ml[i] = (write && c0 + i < nch && c0 + i != own) ? __ldcg(&d.pf_part_ml[prow(c0 + i)])
+                                                               : make_float2(-INFINITY, 0.f);
+          };
+          float Mx = write ? m_used : -INFINITY;
+          load_ml(0);
 #pragma unroll
-              for (int i = 0; i < 32; i += 8)
-                *reinterpret_cast<uint4*>(orow + c * 32 + i) =
-                    make_uint4(pack_bf16(acc[i], acc[i + 1]), pack_bf16(acc[i + 2], acc[i + 3]),
-                               pack_bf16(acc[i + 4], acc[i + 5]),
-                               pack_bf16(acc[i + 6], acc[i + 7]));
+          for (int i = 0; i < MB; ++i) Mx = fmaxf(Mx, ml[i].x);
+          const float ml_f0_x = f0 < MB ? (f0 == 0 ? ml[0].x : ml[1].x) : -INFINITY;
+          float Ls = 0.f;
+#pragma unroll
+          for (int i = 0; i < MB; ++i) Ls += ml[i].y * exp2_safe(ml[i].x, Mx);
+          for (int c0 = MB; c0 < nch; c0 += MB) {
+            load_ml(c0);
+#pragma unroll
+            for (int i = 0; i < MB; ++i) Mx = fmaxf(Mx, ml[i].x);
+          }
+          if (nch > MB) {  // the sum again, against the final maximum
+            Ls = 0.f;
+            for (int c0 = 0; c0 < nch; c0 += MB) {
+              load_ml(c0);
+#pragma unroll
+              for (int i = 0; i < MB; ++i) Ls += ml[i].y * exp2_safe(ml[i].x, Mx);
             }
           }
+          if (write) Ls += l * exp2_safe(m_used, Mx);
+          const float invL = write ? 1.f / Ls : 0.f;
+          const float s_own = write ? exp2_safe(m_used, Mx) : 0.f;
+          // Own part scaled, plus the first other part.
+          float s_f = write ? exp2_safe(ml_f0_x, Mx) : 0.f;
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld32(trow + O_COL + c * 32, o);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const float4 w4 = v[c * 8 + i];
+              o[4 * i] = o[4 * i] * s_own + w4.x * s_f;
+              o[4 * i + 1] = o[4 * i + 1] * s_own + w4.y * s_f;
+              o[4 * i + 2] = o[4 * i + 2] * s_own + w4.z * s_f;
+              o[4 * i + 3] = o[4 * i + 3] * s_own + w4.w * s_f;
+            }
+            tmem_st32(trow + O_COL + c * 32, o);
+          }
+          // The remaining parts (pairs over three or more CTAs), one row at a time.
+          for (int ch = f0 + 1; ch < nch; ++ch) {
+            if (ch == own) continue;
+            load_row(ch, v);
+            s_f = write ? exp2_safe(__ldcg(&d.pf_part_ml[prow(ch)]).x, Mx) : 0.f;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+              float o[32];
+              tmem_ld32(trow + O_COL + c * 32, o);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                const float4 w4 = v[c * 8 + i];
+                o[4 * i] += w4.x * s_f;
+                o[4 * i + 1] += w4.y * s_f;
+                o[4 * i + 2] += w4.z * s_f;
+                o[4 * i + 3] += w4.w * s_f;
+              }
+              tmem_st32(trow + O_COL + c * 32, o);
+            }
+          }
+          __nv_bfloat16* orow = out + ((size_t)(si.q_row0 + t) * d.q_heads + head * G + g) * D;
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld32(trow + O_COL + c * 32, o);
+            if (write) {
+#pragma unroll
+              for (int i = 0; i < 32; i += 8)
+                *reinterpret_cast<uint4*>(orow + c * 32 + i) = make_uint4(
+                    pack_bf16(o[i] * invL, o[i + 1] * invL), pack_bf16(o[i + 2] * invL, o[i + 3] * invL),
+                    pack_bf16(o[i + 4] * invL, o[i + 5] * invL),
+                    pack_bf16(o[i + 6] * invL, o[i + 7] * invL));
+            }
+          }
+          tc_fence_before();
           if (warp == 2 && lane == 0) d.pf_count[seg.seq * H + head] = 0;
         }
       }
