@@ -35,7 +35,7 @@ constexpr int G = 4;
 constexpr int D = 128;
 constexpr int M = 128;                       // MMA rows (query rows, padded)
 constexpr int NK = 64;                       // keys per stage (4 pages)
-constexpr int TC_STAGES = 7;                 // K/V stages: all of shared memory
+constexpr int TC_STAGES = 6;                 // K/V stages of the ring (a 7-stage ring measured slower)
 constexpr int KV_PANEL = NK * 128;           // 64 rows x 128 B = 8 KiB
 constexpr int STAGE = 4 * KV_PANEL;          // K lo, K hi, V lo, V hi = 32 KiB
 // Tensor memory (512 columns x 128 lanes of 32 bits; lane = query row):
