@@ -398,11 +398,14 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
-    # Inputs move on a copy stream, one step ahead of the compute: step i+1's copies are
-    # enqueued just before step i's launches, and each step's compute waits only for its
-    # own inputs, so transfers overlap the previous step's compute.  Results come back on
-    # a third stream, each after an event behind the call that wrote it, so the compute
-    # stream never queues behind a copy.
+    # Inputs move on a copy stream, AHEAD steps ahead of the compute: step i+AHEAD's copies
+    # are enqueued just before step i's launches, and each step's compute waits only for
+    # its own inputs, so transfers overlap earlier steps' compute (the host runs at most a
+    # bounded number of launches ahead of the device, so copies enqueued one step ahead can
+    # start too late on a slow host link).  Results come back on a third stream, each
+    # after an event behind the call that wrote it, so the compute stream never queues
+    # behind a copy.
+    AHEAD = 2
     copy_stream = torch.cuda.Stream()
     d2h_stream = torch.cuda.Stream()
     copy_start = [torch.cuda.Event(enable_timing=True) for _ in steps]
@@ -426,10 +429,11 @@ def run_e2e(drv, w, n_steps: int, world: int, per_layer: bool = False) -> dict:
                     h2d_total += t.numel() * t.element_size()
             ready[si].record(copy_stream)
 
-    enqueue_copies(0)
+    for si in range(min(AHEAD, len(steps))):
+        enqueue_copies(si)
     for si, st in enumerate(steps):
-        if si + 1 < len(steps):
-            enqueue_copies(si + 1)
+        if si + AHEAD < len(steps):
+            enqueue_copies(si + AHEAD)
         stream.wait_event(ready[si])
         comp[si][0].record(stream)
         for ci, c in enumerate(st.calls):
