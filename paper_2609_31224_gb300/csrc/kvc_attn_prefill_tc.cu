@@ -243,6 +243,29 @@ __device__ inline float ex2(float x) {
   return y;
 }
 
+// The segment after `s` in a range ending at u_end, given s.end < u_end: s then ends
+// at its pair's end, and the next segment is the next pair from its first unit, the
+// session's next KV head or the next session's first one.  Unlike unit_segment, no
+// search over the sessions (a chain of dependent loads) is needed.
+__device__ inline UnitSeg next_segment(const Dev& d, const UnitSeg& s, int u_end) {
+  UnitSeg n;
+  if (s.head + 1 < d.kv_heads) {
+    n.seq = s.seq;
+    n.si = s.si;
+    n.head = s.head + 1;
+  } else {
+    n.seq = s.seq + 1;
+    n.si = d.seq[n.seq];
+    n.head = 0;
+  }
+  const int nb = n.si.n_blocks;
+  n.pair_start = n.si.unit_base + n.head * nb;
+  n.pair_end = n.pair_start + nb;
+  n.u = s.end;
+  n.end = min(u_end, n.pair_end);
+  return n;
+}
+
 // FUSED (the per-layer order): the chunk's K (rotated at each token's position) and
 // V of this layer are not in the pool yet; new_k / new_v hold them ([total][Hkv][D],
 // the append's token order).  The producer warp that loads a stage holding chunk
@@ -322,8 +345,9 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
     bool stop = false;
     uint32_t rows_seen = 0;  // segments holding chunk slots, before this one
     (void)rows_seen;
+    UnitSeg seg;
     for (int u = u_begin; u < u_end && !stop;) {
-      const UnitSeg seg = unit_segment(d, u, u_end);
+      seg = u == u_begin ? unit_segment(d, u, u_end) : next_segment(d, seg, u_end);
       u = seg.end;
       const int head = seg.head;
       const SeqInfo& si = seg.si;
@@ -410,8 +434,9 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
         constexpr uint32_t ID_S = instr_desc(NK, M, false);
         uint32_t sc = 0;     // S tiles issued
         uint32_t segs = 0;   // segments started
+        UnitSeg seg;
         for (int u = u_begin; u < u_end && !s_abort; ++segs) {
-          const UnitSeg seg = unit_segment(d, u, u_end);
+          seg = u == u_begin ? unit_segment(d, u, u_end) : next_segment(d, seg, u_end);
           u = seg.end;
           const int n_st = (seg.end - seg.u + 3) / 4;
           if (!mbar_wait(d, &bars[B_Q], segs & 1)) {
@@ -445,8 +470,9 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       } else {
         constexpr uint32_t ID_PV = instr_desc(D, M, true);
         uint32_t pv = 0;  // P V products issued
+        UnitSeg seg;
         for (int u = u_begin; u < u_end && !s_abort;) {
-          const UnitSeg seg = unit_segment(d, u, u_end);
+          seg = u == u_begin ? unit_segment(d, u, u_end) : next_segment(d, seg, u_end);
           u = seg.end;
           const int n_st = (seg.end - seg.u + 3) / 4;
           for (int k = 0; k < n_st && !s_abort; ++k) {
@@ -496,8 +522,9 @@ __global__ void __launch_bounds__(THREADS, 1) attn_prefill_tc_kernel(
       dead = !__all_sync(FULL, mbar_wait(d, bar, parity));
       if (dead && lane == 0) s_abort = 1;
     };
+    UnitSeg seg;
     for (int u = u_begin; u < u_end;) {
-      const UnitSeg seg = unit_segment(d, u, u_end);
+      seg = u == u_begin ? unit_segment(d, u, u_end) : next_segment(d, seg, u_end);
       const int first = seg.u == u_begin;
       u = seg.end;
       const int head = seg.head;
