@@ -37,15 +37,16 @@ UNIT = "audio-s/s"
 
 
 # DRAM bytes per algorithmic byte of the roofline kernel (reads + writes), from one
-# ncu capture of the stream-K kernel on the 24-session, two-layer reduced case:
-# 409.79 MB of traffic (406.83 MB read, 2.97 MB written) for a 403.97 MB launch.  Valid only
-# while the decode sources hash to the version it was taken on; the roofline's traffic is
-# null otherwise.
-DECODE_TRAFFIC_RATIO = 409.79 / 403.97
+# ncu capture of the stream-K kernel on the 64-session, two-layer case (the bench's
+# launch shape; smaller calls run the pair-split kernel): 1,088.24 MB of traffic
+# (1,084.54 MB read, 3.70 MB written) for a 1,077.10 MB launch.  Valid only while the
+# decode sources hash to the version it was taken on; the roofline's traffic is null
+# otherwise.
+DECODE_TRAFFIC_RATIO = 1088.24 / 1077.10
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
                           "paper_2609_31224_gb300/csrc/kvc_decode_common.cuh",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "463ff4e942d77aeda9e12db0da7a1ddc1b0243ecdbefce712a590c92d790e1d4"
+DECODE_TRAFFIC_SHA256 = "287ae340f59f9a1522acce9f04e2c9e0e753da584dcf073b9bdf4196369b20f7"
 
 
 def decode_traffic(alg_bytes_per_launch):
@@ -64,14 +65,14 @@ def decode_traffic(alg_bytes_per_launch):
 def decode_kernel_label(w) -> str:
     """Kernel that the library's dispatch gives a full-batch decode call of `w` (sessions
     at full budget): the 16-warp pair split while every (session, KV head) pair gets two
-    one-CTA-per-SM slices, the 4-warp pair split while it gets three of the three CTAs
-    per SM, else stream-K."""
+    one-CTA-per-SM slices, the 4-warp pair split while it gets one of the three CTAs per
+    SM, else stream-K."""
     import torch
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     pairs = w.n_sessions * w.kv_heads
     if 2 * pairs <= sms:
         return "attn_decode_split_kernel (16 warps)"
-    if pairs <= sms:
+    if pairs <= 3 * sms:
         return "attn_decode_split_kernel (4 warps)"
     return "attn_decode_kernel"
 
@@ -358,7 +359,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "frac": (dec_gbs / peak) if dec_gbs else None,
             "traffic": decode_traffic((sum(dec_bytes) / len(dec_bytes)) if dec_bytes else None),
             "traffic_note": "ncu DRAM bytes per algorithmic byte of the stream-K kernel on "
-                            "the 24-session reduced case, scaled to this launch",
+                            "the 64-session two-layer case, times this launch's bytes",
             "algorithmic_bytes_per_launch": (sum(dec_bytes) / len(dec_bytes)) if dec_bytes else None,
             "avg_launch_us": (1e3 * sum(dec_times) / len(dec_times)) if dec_times else None,
         },

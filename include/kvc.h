@@ -234,9 +234,9 @@ int kvc_attn_prefill_chunk_kv(kvc_ctx* ctx, int layer, const void* d_k, const vo
  * original rotary positions.  The last append gave each of its n_seq sessions
  * exactly one token; that token attends to every resident key, itself included.
  * Split-K over pages with a log-sum-exp merge.
- * Precision depends on the call's size: for bfloat16 calls of at most 9 sessions
- * (8 KV heads, 152 SMs: while every (session, KV head) pair gets two one-CTA-per-SM
- * slices) the page products run on tensor cores with q and P rounded to bfloat16
+ * Precision depends on the call's size: for bfloat16 calls of at most 57 sessions
+ * (8 KV heads, 152 SMs: while every (session, KV head) pair gets a CTA of its own in
+ * one wave) the page products run on tensor cores with q and P rounded to bfloat16
  * and binary32 accumulation; larger calls keep q and P in binary32 on CUDA cores.
  * So the same session's output can differ in the last bits with the number of
  * sessions sharing its call; both stay within the attention tolerance.

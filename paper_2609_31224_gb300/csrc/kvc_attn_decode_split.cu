@@ -1,10 +1,10 @@
 // Single-token decode attention, pair-split kernel (calls of few sessions): CTA
 // c takes slice c % k of (session, KV head) pair c / k, the pair's pages cut into
-// k equal slices, so that every page of a small call is in flight at once.  With
-// 16 warps (one CTA per SM) the bfloat16 pages run on the tensor cores
-// (mma.sync) and the partial states are tagged 64-bit words merged after a
-// relaxed arrival; with 4 warps (three CTAs per SM) the CUDA-core page loop and
-// the acquire-release arrival of stream-K are used.
+// k equal slices, so that every page of a small call is in flight at once.  The
+// bfloat16 pages run on the tensor cores (mma.sync) in both CTA shapes.  With 16
+// warps (one CTA per SM) the partial states are tagged 64-bit words merged after a
+// relaxed arrival; with 4 warps (three CTAs per SM) the acquire-release arrival of
+// stream-K is used.
 #include "kvc_decode_common.cuh"
 
 // Shape constants of the CUDA-core loop are unused by the tensor-core shapes.

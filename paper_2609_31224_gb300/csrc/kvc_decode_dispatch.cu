@@ -2,8 +2,10 @@
 // kernel shapes, by the number of (session, KV head) pairs it has:
 //   - pair split, 16-warp CTAs (one per SM): every pair gets k >= 2 CTAs in one
 //     wave; for bfloat16 the pages run on the tensor cores;
-//   - pair split, 4-warp CTAs (three per SM): k >= 3;
-//   - stream-K over (session, KV head, page) units: the rest (the full-batch rounds).
+//   - pair split, 4-warp CTAs (three per SM, tensor-core pages for bfloat16): every
+//     pair gets k >= 1 CTAs in one wave (with k = 1 a pair needs no merge);
+//   - stream-K over (session, KV head, page) units: the rest (more pairs than the
+//     4-warp shape's resident CTAs, e.g. the full-batch rounds of 64 sessions).
 #include <cstring>
 
 #include "kvc_launch.cuh"
@@ -19,8 +21,12 @@ constexpr int DEC_MIN_UNITS = 12;
 // The pair-split kernel takes calls whose pairs each get at least this many CTAs
 // in one wave: with 16-warp CTAs (one per SM) first, else with stream-K's 4-warp
 // CTAs (three per SM).  Only the 16-warp shape uses tagged partial states: with
-// 4-warp CTAs the fenced arrival measured faster.
-constexpr int SPLIT_MIN_K = 2, SPLIT4_MIN_K = 3;
+// 4-warp CTAs the fenced arrival measured faster.  Against stream-K (CUDA-core
+// pages), the 4-warp tensor-core split measured faster at 20-28 sessions with two
+// slices per pair (56.1 against 60.8 us at 20, 71.1 against 79.0 at 28) and, with one,
+// at 29-57 sessions except near 36 (73.2 against 81.7 at 29, 99.6 against 97.7 at
+// 36, 138.4 against 148.2 at 57).
+constexpr int SPLIT_MIN_K = 2, SPLIT4_MIN_K = 1;
 
 }  // namespace
 

@@ -62,7 +62,9 @@ def test_the_committed_traffic_ratio_matches_the_committed_sources():
     (9, "attn_decode_split_kernel (16 warps)"),
     (10, "attn_decode_split_kernel (4 warps)"),
     (19, "attn_decode_split_kernel (4 warps)"),
-    (20, "attn_decode_kernel"),
+    (28, "attn_decode_split_kernel (4 warps)"),
+    (57, "attn_decode_split_kernel (4 warps)"),
+    (58, "attn_decode_kernel"),
     (64, "attn_decode_kernel"),
 ])
 def test_roofline_kernel_label_follows_the_dispatch(sessions, label, monkeypatch):

@@ -349,19 +349,19 @@ def _sms():
 
 def _decode_tier(n_seq, kv_heads):
     """Decode kernel the library dispatches for a call of n_seq sessions: the 16-warp pair
-    split (one CTA per SM, tensor-core pages) while every (session, KV head) pair gets two
-    slices, the 4-warp pair split while it gets three of the three CTAs per SM, else
-    stream-K."""
+    split (one CTA per SM) while every (session, KV head) pair gets two slices, the 4-warp
+    pair split while it gets one of the three CTAs per SM, else stream-K."""
     pairs = n_seq * kv_heads
     if 2 * pairs <= _sms():
         return "split16"
-    if 3 * pairs <= 3 * _sms():
+    if pairs <= 3 * _sms():
         return "split4"
     return "streamk"
 
 
 def test_decode_4warp_tier_at_full_budget():
-    """Decode calls of 10-19 sessions (the 4-warp pair split on 152 SMs) at full budget,
+    """Decode calls of 10-19 sessions (the 4-warp pair split with three slices or more per
+    pair on 152 SMs) at full budget,
     every output of every session compared with the oracle: the first two natural decode
     rounds of that size in a step of a 19-session shard of the 64-session workload at its
     steady state, then calls of exactly 10, 12, 16 and 19 sessions (one transcript token
@@ -400,12 +400,36 @@ def test_decode_4warp_tier_at_full_budget():
     assert ls.n_compared >= 10 * 2 + 12 + 16 + 19
 
 
+def test_decode_4warp_tier_one_and_two_slices():
+    """Decode calls of 20-57 sessions, where the 4-warp pair split gives every (session, KV
+    head) pair two slices (20-28 sessions, merged by the last to arrive) or one (29-57, no
+    merge), at full budget: a 57-session shard of the 64-session workload brought to its
+    steady state, then calls of exactly 20, 28, 29, 40 and 57 sessions (one transcript
+    token each), every output of layer 0 compared with the oracle."""
+    w = S.BATCH64_BF16
+    scripts = S.workload_scripts(w)
+    shard = sorted(scripts, key=lambda sc: sc.offset)[:57]
+    drv = Driver(w, shard)
+    ls = Lockstep(drv, w)
+    steady = S.steady_state_step(w, shard)
+    for _ in range(steady):
+        ls.run_step(check_state=False)
+    for n in (20, 28, 29, 40, 57):
+        ls.decode_call([sc.session for sc in shard[:n]], layers=(0,))
+        if _sms() == 152:
+            assert _decode_tier(n, w.kv_heads) == "split4"
+    for sc in shard[:20]:
+        st = drv.cache.export_state(sc.session)
+        assert st["resident"] >= 4000 and st["n_evicted"] > 0
+    assert ls.n_compared >= 20 + 28 + 29 + 40 + 57
+
+
 def test_batch64_sampled_at_full_size():
     """64 sessions, offsets U{0..300}, run through the benchmark's timed window (its 20
     steps from the steady state): the state of every session bit-exact at sampled steps and
     after every evict of the window; attention in the benchmark's launch configuration at
     three steps of the window: the prefill call and the first decode round of each kernel
-    tier present (stream-K for >= 20 sessions, the 4-warp pair split for 10-19, the
+    tier present (stream-K for >= 58 sessions, the 4-warp pair split for 10-57, the
     16-warp tensor-core pair split for <= 9, and a one-session round)."""
     w = S.BATCH64_BF16
     scripts = S.workload_scripts(w)
