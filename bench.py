@@ -64,13 +64,13 @@ def decode_traffic(alg_bytes_per_launch):
 
 def decode_kernel_label(w) -> str:
     """Kernel that the library's dispatch gives a full-batch decode call of `w` (sessions
-    at full budget): the 16-warp pair split while every (session, KV head) pair gets two
+    at full budget): the 16-warp pair split while every (session, KV head) pair gets five
     one-CTA-per-SM slices, the 4-warp pair split while it gets one of the three CTAs per
     SM, else stream-K."""
     import torch
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     pairs = w.n_sessions * w.kv_heads
-    if 2 * pairs <= sms:
+    if 5 * pairs <= sms:
         return "attn_decode_split_kernel (16 warps)"
     if pairs <= 3 * sms:
         return "attn_decode_split_kernel (4 warps)"

@@ -1,7 +1,8 @@
 // Dispatch of a decode attention call (one token per session) between the three
 // kernel shapes, by the number of (session, KV head) pairs it has:
-//   - pair split, 16-warp CTAs (one per SM): every pair gets k >= 2 CTAs in one
-//     wave; for bfloat16 the pages run on the tensor cores;
+//   - pair split, 16-warp CTAs (one per SM): every pair gets k >= 5 CTAs in one
+//     wave (at most 3 sessions of 8 KV heads on 152 SMs); for bfloat16 the pages run
+//     on the tensor cores;
 //   - pair split, 4-warp CTAs (three per SM, tensor-core pages for bfloat16): every
 //     pair gets k >= 1 CTAs in one wave (with k = 1 a pair needs no merge);
 //   - stream-K over (session, KV head, page) units: the rest (more pairs than the
@@ -25,8 +26,10 @@ constexpr int DEC_MIN_UNITS = 12;
 // pages), the 4-warp tensor-core split measured faster at 20-28 sessions with two
 // slices per pair (56.1 against 60.8 us at 20, 71.1 against 79.0 at 28) and, with one,
 // at 29-57 sessions except near 36 (73.2 against 81.7 at 29, 99.6 against 97.7 at
-// 36, 138.4 against 148.2 at 57).
-constexpr int SPLIT_MIN_K = 2, SPLIT4_MIN_K = 1;
+// 36, 138.4 against 148.2 at 57).  Against the 16-warp shape, the 4-warp one measured
+// faster from 4 sessions on (15.4 against 16.7 us at 4, 26.4 against 28.1 at 9) and
+// slower below (11.7 against 8.1 at 1).
+constexpr int SPLIT_MIN_K = 5, SPLIT4_MIN_K = 1;
 
 }  // namespace
 

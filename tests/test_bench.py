@@ -59,7 +59,9 @@ def test_the_committed_traffic_ratio_matches_the_committed_sources():
 
 @pytest.mark.parametrize("sessions,label", [
     (1, "attn_decode_split_kernel (16 warps)"),
-    (9, "attn_decode_split_kernel (16 warps)"),
+    (3, "attn_decode_split_kernel (16 warps)"),
+    (4, "attn_decode_split_kernel (4 warps)"),
+    (9, "attn_decode_split_kernel (4 warps)"),
     (10, "attn_decode_split_kernel (4 warps)"),
     (19, "attn_decode_split_kernel (4 warps)"),
     (28, "attn_decode_split_kernel (4 warps)"),

@@ -349,10 +349,10 @@ def _sms():
 
 def _decode_tier(n_seq, kv_heads):
     """Decode kernel the library dispatches for a call of n_seq sessions: the 16-warp pair
-    split (one CTA per SM) while every (session, KV head) pair gets two slices, the 4-warp
+    split (one CTA per SM) while every (session, KV head) pair gets five slices, the 4-warp
     pair split while it gets one of the three CTAs per SM, else stream-K."""
     pairs = n_seq * kv_heads
-    if 2 * pairs <= _sms():
+    if 5 * pairs <= _sms():
         return "split16"
     if pairs <= 3 * _sms():
         return "split4"
@@ -429,8 +429,8 @@ def test_batch64_sampled_at_full_size():
     steps from the steady state): the state of every session bit-exact at sampled steps and
     after every evict of the window; attention in the benchmark's launch configuration at
     three steps of the window: the prefill call and the first decode round of each kernel
-    tier present (stream-K for >= 58 sessions, the 4-warp pair split for 10-57, the
-    16-warp tensor-core pair split for <= 9, and a one-session round)."""
+    tier present (stream-K for >= 58 sessions, the 4-warp pair split for 4-57, the
+    16-warp tensor-core pair split for <= 3, and a one-session round)."""
     w = S.BATCH64_BF16
     scripts = S.workload_scripts(w)
     drv = Driver(w, scripts)
