@@ -38,15 +38,15 @@ UNIT = "audio-s/s"
 
 # DRAM bytes per algorithmic byte of the roofline kernel (reads + writes), from one
 # ncu capture of the stream-K kernel on the 64-session, two-layer case (the bench's
-# launch shape; smaller calls run the pair-split kernel): 1,088.24 MB of traffic
-# (1,084.54 MB read, 3.70 MB written) for a 1,077.10 MB launch.  Valid only while the
+# launch shape; smaller calls run the pair-split kernel): 1,088.57 MB of traffic
+# (1,084.41 MB read, 4.16 MB written) for a 1,077.10 MB launch.  Valid only while the
 # decode sources hash to the version it was taken on; the roofline's traffic is null
 # otherwise.
-DECODE_TRAFFIC_RATIO = 1088.24 / 1077.10
+DECODE_TRAFFIC_RATIO = 1088.57 / 1077.10
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
                           "paper_2609_31224_gb300/csrc/kvc_decode_common.cuh",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "287ae340f59f9a1522acce9f04e2c9e0e753da584dcf073b9bdf4196369b20f7"
+DECODE_TRAFFIC_SHA256 = "8057e231d2b9b2f3b8f9c0ff3156dc61e0204c15e89e2bea6c1c00cdf064823e"
 
 
 def decode_traffic(alg_bytes_per_launch):

@@ -234,12 +234,12 @@ int kvc_attn_prefill_chunk_kv(kvc_ctx* ctx, int layer, const void* d_k, const vo
  * original rotary positions.  The last append gave each of its n_seq sessions
  * exactly one token; that token attends to every resident key, itself included.
  * Split-K over pages with a log-sum-exp merge.
- * Precision depends on the call's size: for bfloat16 calls of at most 57 sessions
- * (8 KV heads, 152 SMs: while every (session, KV head) pair gets a CTA of its own in
- * one wave) the page products run on tensor cores with q and P rounded to bfloat16
- * and binary32 accumulation; larger calls keep q and P in binary32 on CUDA cores.
- * So the same session's output can differ in the last bits with the number of
- * sessions sharing its call; both stay within the attention tolerance.
+ * Precision: for bfloat16 the page products run on tensor cores with q and P
+ * rounded to bfloat16 and binary32 accumulation and softmax, in every call size;
+ * binary32 calls run on CUDA cores in binary32.  The split of a session's pages
+ * over CTAs (and so the order of the partial sums) depends on how many sessions
+ * share its call, so its output can differ in the last bits with that number;
+ * both stay within the attention tolerance.
  *   d_q     device [n_seq][Hq][D] un-rotated queries (call order of the append)
  *   d_out   device [n_seq][Hq][D]
  * May be captured into a CUDA graph: a launch made while `stream` is capturing

@@ -40,7 +40,6 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
     const __grid_constant__ CUtensorMap map_hi, const T* __restrict__ q, T* __restrict__ out,
     float qk_scale, int min_units, const T* new_k, const T* new_v) {
   using C = SkCfg<T, D>;
-  static_assert(!C::MMA, "the stream-K kernel runs the CUDA-core page loop");
   static_assert(C::WARPS == G, "the split-K merge maps one warp to one query row");
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -70,23 +69,36 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
     const int pair_start = seg.pair_start, pair_end = seg.pair_end, seg_end = seg.end;
 
     Segment<C> sg;
-    sg.init(d, si, head, u - pair_start, seg_end - u, warp);
+    sg.init(d, si, head, u - pair_start, seg_end - u, warp, &map_lo, &map_hi);
     sg.prefetch(d, layer, sm, loads, warp, lane);
     if (!waited) {
       if (warp == 0) prefetch_q<C>(d, si, head, q, lane);
       pdl_wait();
       waited = true;
     }
-    float qr[G][2 * C::VEC];
-    load_q<C>(d, si, head, q, qk_scale, lane, qr);
+    int failed_at;
+    // The page loop's state: tensor-core fragments (bfloat16) or CUDA-core rows.
+    float m2[2] = {-INFINITY, -INFINITY}, l2[2] = {0.f, 0.f};
+    float o[8][4];
     float m_run = -INFINITY, l_run = 0.f;  // for row lane >> 3
     float2 acc[G][C::PVD / 2];
+    if constexpr (C::MMA) {
+      uint32_t qb[8][2];
+      load_q_mma<C>(d, si, head, q, qk_scale, lane, qb);
 #pragma unroll
-    for (int g = 0; g < G; ++g)
+      for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+      failed_at = stream_pages_mma<C, FUSED>(d, layer, sg, sm, loads, qb, m2, l2, o, warp, lane,
+                                             new_k, new_v);
+    } else {
+      float qr[G][2 * C::VEC];
+      load_q<C>(d, si, head, q, qk_scale, lane, qr);
 #pragma unroll
-      for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
-    const int failed_at = stream_pages<C, FUSED>(d, layer, sg, sm, loads, qr, m_run, l_run, acc,
-                                                 warp, lane, new_k, new_v);
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int j = 0; j < C::PVD / 2; ++j) acc[g][j] = make_float2(0.f, 0.f);
+      failed_at = stream_pages<C, FUSED>(d, layer, sg, sm, loads, qr, m_run, l_run, acc, warp,
+                                         lane, new_k, new_v);
+    }
     if (failed_at >= 0 && lane == 0) s_abort = 1;
     __syncthreads();
     if (s_abort) {
@@ -103,7 +115,10 @@ __global__ void __launch_bounds__(SkCfg<T, D>::THREADS) attn_decode_kernel(
     loads += sg.n_my;
 
     // Merge the four warps' partial softmax states (stage buffers are free now).
-    publish_warp<C>(sm, m_run, l_run, acc, warp, lane);
+    if constexpr (C::MMA)
+      publish_warp_mma<C>(sm, m2, l2, o, warp, lane);
+    else
+      publish_warp<C>(sm, m_run, l_run, acc, warp, lane);
     __syncthreads();
     merge_warps<C>(sm, warp, lane);
     const bool whole = u == pair_start && seg_end == pair_end;

@@ -45,9 +45,9 @@ struct DecCfg {
 };
 
 // Stream-K kernel: 4 warps (one per query row in the split-K merge), 2-deep rings,
-// three CTAs per SM.
+// three CTAs per SM; tensor-core pages for bfloat16.
 template <typename T, int D>
-using SkCfg = DecCfg<T, D, 4, 2>;
+using SkCfg = DecCfg<T, D, 4, 2, true>;
 // Pair-split kernel: 16 warps, one tile pair each, one CTA per SM; with few
 // sessions every page of the call is in flight at once.  Its pages are latency-
 // bound, so for bfloat16 they run on the tensor cores (fewer instructions per page).
@@ -571,6 +571,219 @@ __device__ void merge_parts(const Dev& d, const Smem<C>& sm, int nch, PartFn par
   for (int t = 0; t < EPT; ++t) {
     const int e = tid + t * C::THREADS;
     if (e < G * D) orow[e] = from_float<T>(O[t]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Tensor-core page loop (bfloat16, D = 128).  Per page of 16 keys and the G = 4
+// query rows of one KV head, with the keys as the MMA's M dimension:
+//   S^T [16 keys x 8 rows]  = K [16 x 128] . Q^T [128 x 8]        (8 k-steps)
+//   O^T [128 dims x 8 rows] += V^T [128 x 16 keys] . P^T [16 x 8]  (8 m-tiles)
+// with mma.sync m16n8k16 (bf16 in, fp32 accumulate); rows 4..7 are zero padding.
+// Lane (g, t) = (lane >> 2, lane & 3) holds S^T for keys g, g + 8 and rows 2t,
+// 2t + 1, so it owns the softmax state of rows 2t, 2t + 1 (valid for t < 2), and
+// O^T for dims 16 mt + g (+ 8) of the same rows.  Tiles are two 64-column boxes
+// (2 KiB, 16 rows of 128 B) with the 128-byte swizzle: 16-byte chunk c of row r
+// sits at chunk c ^ (r & 7), so ldmatrix reads of 8 rows hit 8 distinct banks.
+// ---------------------------------------------------------------------------
+__device__ inline uint32_t swz(int row, int col) {  // col: a multiple of 8 in [0, 128)
+  return (col >> 6) * 2048 + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4);
+}
+
+__device__ inline void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ inline void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ inline void mma_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                 uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ inline uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// Query rows of `head`, rotated at the token's position, scaled by log2(e)/sqrt(D)
+// and rounded to bfloat16, as the B operand Q^T of the score products: lane (g, t)
+// with g < G holds dims 16 ks + 2t, +1 (qb[ks][0]) and 16 ks + 2t + 8, +9
+// (qb[ks][1]) of row g; lanes g >= G hold the zero rows.  Dims d and d + 64 (k-steps
+// ks and ks + 4 of the same lane) are rotated together.
+template <class C>
+__device__ void load_q_mma(const Dev& d, const SeqInfo& si, int head, const typename C::T* q,
+                           float qk_scale, int lane, uint32_t (&qb)[8][2]) {
+  static_assert(C::D == 128, "tensor-core page loop assumes D = 128");
+  const int g = lane >> 2, t = lane & 3;
+  if (g >= G) {
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) qb[ks][0] = qb[ks][1] = 0u;
+    return;
+  }
+  const uint32_t* qrow = reinterpret_cast<const uint32_t*>(
+      q + ((size_t)si.q_row0 * d.q_heads + (size_t)head * G + g) * C::D);
+  const float2* cs = d.rope + (size_t)si.pos_first * (C::D / 2);
+  uint32_t w[8][2];
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    w[ks][0] = qrow[8 * ks + t];
+    w[ks][1] = qrow[8 * ks + t + 4];
+  }
+  float2 c[4][4];
+#pragma unroll
+  for (int ks = 0; ks < 4; ++ks)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      c[ks][2 * j] = cs[16 * ks + 2 * t + 8 * j];
+      c[ks][2 * j + 1] = cs[16 * ks + 2 * t + 8 * j + 1];
+    }
+#pragma unroll
+  for (int ks = 0; ks < 4; ++ks)
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const float x0 = bf16lo(w[ks][j]), x1 = bf16hi(w[ks][j]);          // dims < 64
+      const float y0 = bf16lo(w[ks + 4][j]), y1 = bf16hi(w[ks + 4][j]);  // dims + 64
+      const float2 c0 = c[ks][2 * j], c1 = c[ks][2 * j + 1];
+      qb[ks][j] = pack_bf16x2(fmaf(x0, c0.x, -y0 * c0.y) * qk_scale,
+                              fmaf(x1, c1.x, -y1 * c1.y) * qk_scale);
+      qb[ks + 4][j] = pack_bf16x2(fmaf(y0, c0.x, x0 * c0.y) * qk_scale,
+                                  fmaf(y1, c1.x, x1 * c1.y) * qk_scale);
+    }
+}
+
+// stream_pages on the tensor cores.  m_run / l_run: running max and this lane's
+// partial sum of rows 2t, 2t + 1 (the sum is completed over g by publish_warp_mma).
+template <class C, bool FUSED>
+__device__ int stream_pages_mma(const Dev& d, int layer, Segment<C>& sg, const Smem<C>& sm,
+                                uint32_t loads, const uint32_t (&qb)[8][2], float (&m_run)[2],
+                                float (&l_run)[2], float (&o)[8][4], int warp, int lane,
+                                const typename C::T* new_k, const typename C::T* new_v) {
+  const int g = lane >> 2, t = lane & 3;
+  // ldmatrix row of this lane: K (A = K, keys x dims) and V (A = V^T via .trans).
+  const int k_key = (lane & 7) + 8 * ((lane >> 3) & 1), k_col = 8 * (lane >> 4);
+  const int v_key = (lane & 7) + 8 * (lane >> 4), v_col = 8 * ((lane >> 3) & 1);
+  __nv_bfloat16* pt = reinterpret_cast<__nv_bfloat16*>(sm.s_sc);  // P^T as [G][PS]
+  for (int k = 0; k < sg.n_my; ++k) {
+    const uint32_t n = loads + k;
+    const int st = n % C::STAGES;
+    if (!__all_sync(FULL, mbar_wait(d, &sm.wbars[st], (n / C::STAGES) & 1))) return k;
+    uint8_t* kt = sm.tiles + st * 2 * C::TILE;
+    const int blk = sg.blk_begin + warp + k * C::WARPS;
+    if constexpr (FUSED) {
+      if (blk == sg.si.n_blocks - 1)
+        patch_new_row<C>(d, layer, sg.si, sg.head, new_k, new_v, kt, lane);
+    }
+    const uint32_t kb = smem_u32(kt), vb = kb + C::TILE;
+
+    float s[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      uint32_t a[4];
+      ldsm_x4(a, kb + swz(k_key, 16 * ks + k_col));
+      mma_16816(s, a, qb[ks][0], qb[ks][1]);
+    }
+    const BlockRange br = block_range(sg.si, blk);
+    if (!(br.lo == 0 && br.hi == PS)) {
+      if (g < br.lo || g >= br.hi) s[0] = s[1] = -INFINITY;
+      if (g + 8 < br.lo || g + 8 >= br.hi) s[2] = s[3] = -INFINITY;
+    }
+    // Online softmax of rows 2t (s0, s2) and 2t + 1 (s1, s3) over the page's keys.
+    float mx0 = fmaxf(s[0], s[2]), mx1 = fmaxf(s[1], s[3]);
+#pragma unroll
+    for (int off = 4; off < 32; off <<= 1) {
+      mx0 = fmaxf(mx0, __shfl_xor_sync(FULL, mx0, off));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(FULL, mx1, off));
+    }
+    const float mn0 = fmaxf(m_run[0], mx0), mn1 = fmaxf(m_run[1], mx1);
+    const float p0 = exp2_safe(s[0], mn0), p2 = exp2_safe(s[2], mn0);
+    const float p1 = exp2_safe(s[1], mn1), p3 = exp2_safe(s[3], mn1);
+    const float al0 = exp2_safe(m_run[0], mn0), al1 = exp2_safe(m_run[1], mn1);
+    l_run[0] = l_run[0] * al0 + (p0 + p2);
+    l_run[1] = l_run[1] * al1 + (p1 + p3);
+    m_run[0] = mn0;
+    m_run[1] = mn1;
+    // P^T to the B-operand layout through shared memory: lane (g, t < 2) writes
+    // P[row][key] for its two rows and keys g, g + 8; lane (g < G, t) reads keys
+    // 2t, 2t + 1 and 2t + 8, 2t + 9 of row g.
+    __syncwarp();
+    if (t < 2) {
+      pt[(2 * t) * PS + g] = __float2bfloat16_rn(p0);
+      pt[(2 * t + 1) * PS + g] = __float2bfloat16_rn(p1);
+      pt[(2 * t) * PS + g + 8] = __float2bfloat16_rn(p2);
+      pt[(2 * t + 1) * PS + g + 8] = __float2bfloat16_rn(p3);
+    }
+    __syncwarp();
+    uint32_t pb0 = 0u, pb1 = 0u;
+    if (g < G) {
+      pb0 = *reinterpret_cast<const uint32_t*>(pt + g * PS + 2 * t);
+      pb1 = *reinterpret_cast<const uint32_t*>(pt + g * PS + 2 * t + 8);
+    }
+    if (__any_sync(FULL, al0 != 1.f || al1 != 1.f)) {
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        o[mt][0] *= al0;
+        o[mt][1] *= al1;
+        o[mt][2] *= al0;
+        o[mt][3] *= al1;
+      }
+    }
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      uint32_t a[4];
+      ldsm_x4_trans(a, vb + swz(v_key, 16 * mt + v_col));
+      mma_16816(o[mt], a, pb0, pb1);
+    }
+    __syncwarp();
+    if (k + C::STAGES < sg.n_my) {
+      if (lane == 0) fence_proxy_async_smem();
+      sg.issue(d, layer, sm, loads, k + C::STAGES, warp, lane);
+    }
+  }
+  return -1;
+}
+
+// publish_warp for the tensor-core state: completes each row's sum over the lanes
+// holding its keys and writes (m, l) and the row's unnormalised output.
+template <class C>
+__device__ void publish_warp_mma(const Smem<C>& sm, const float (&m_run)[2],
+                                 const float (&l_run)[2], const float (&o)[8][4], int warp,
+                                 int lane) {
+  constexpr int D = C::D;
+  const int g = lane >> 2, t = lane & 3;
+  float l0 = l_run[0], l1 = l_run[1];
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    l0 += __shfl_xor_sync(FULL, l0, off);
+    l1 += __shfl_xor_sync(FULL, l1, off);
+  }
+  if (t < 2) {
+    const int r0 = warp * G + 2 * t, r1 = r0 + 1;
+    if (g == 0) {
+      sm.m_ml[r0 * 2 + 0] = m_run[0];
+      sm.m_ml[r0 * 2 + 1] = l0;
+      sm.m_ml[r1 * 2 + 0] = m_run[1];
+      sm.m_ml[r1 * 2 + 1] = l1;
+    }
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+      sm.m_o[r0 * D + 16 * mt + g] = o[mt][0];
+      sm.m_o[r1 * D + 16 * mt + g] = o[mt][1];
+      sm.m_o[r0 * D + 16 * mt + g + 8] = o[mt][2];
+      sm.m_o[r1 * D + 16 * mt + g + 8] = o[mt][3];
+    }
   }
 }
 

@@ -5,8 +5,9 @@
 //     on the tensor cores;
 //   - pair split, 4-warp CTAs (three per SM, tensor-core pages for bfloat16): every
 //     pair gets k >= 1 CTAs in one wave (with k = 1 a pair needs no merge);
-//   - stream-K over (session, KV head, page) units: the rest (more pairs than the
-//     4-warp shape's resident CTAs, e.g. the full-batch rounds of 64 sessions).
+//   - stream-K over (session, KV head, page) units, tensor-core pages for bfloat16:
+//     the rest (more pairs than the 4-warp shape's resident CTAs, e.g. the full-batch
+//     rounds of 64 sessions).
 #include <cstring>
 
 #include "kvc_launch.cuh"
@@ -58,8 +59,9 @@ cudaError_t launch_attn_decode(const Dev& d, int layer, const void* q, void* out
   CUtensorMap map_lo, map_hi;
   memset(&map_lo, 0, sizeof(map_lo));
   memset(&map_hi, 0, sizeof(map_hi));
+  // (The stream-K kernel's bfloat16 pages also run on the tensor cores.)
   if (((k > 0 && decode_split_uses_tma(esz, true)) ||
-       (k4 > 0 && decode_split_uses_tma(esz, false))) &&
+       (k4 > 0 && decode_split_uses_tma(esz, false)) || (k == 0 && k4 == 0 && esz == 2)) &&
       !pool_tensor_maps(d, &map_lo, &map_hi))
     return cudaErrorInvalidValue;
   if (k > 0) {
