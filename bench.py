@@ -19,6 +19,7 @@ from __future__ import annotations
 
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -46,18 +47,31 @@ DECODE_TRAFFIC_RATIO = 1088.57 / 1077.10
 DECODE_TRAFFIC_SOURCES = ("paper_2609_31224_gb300/csrc/kvc_attn_decode.cu",
                           "paper_2609_31224_gb300/csrc/kvc_decode_common.cuh",
                           "paper_2609_31224_gb300/csrc/kvc_internal.cuh")
-DECODE_TRAFFIC_SHA256 = "8057e231d2b9b2f3b8f9c0ff3156dc61e0204c15e89e2bea6c1c00cdf064823e"
+DECODE_TRAFFIC_SHA256 = "1e7582c380f739e8b63919fc568b9687161723d1076652b086603f3e9759a8e7"
+
+
+def code_only(text: str) -> str:
+    """C/C++ source without its comments and with whitespace collapsed: what the compiler
+    sees of it (the decode sources hold no string literal with a comment marker)."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
+def decode_sources_digest(root: str | None = None) -> str:
+    """SHA-256 of the decode sources' code (comments and layout excluded)."""
+    h = hashlib.sha256()
+    for f in DECODE_TRAFFIC_SOURCES:
+        with open(os.path.join(root or ROOT, f), encoding="utf-8") as fh:
+            h.update(code_only(fh.read()).encode())
+    return h.hexdigest()
 
 
 def decode_traffic(alg_bytes_per_launch):
     """Per-launch DRAM traffic of the decode kernel, scaled from the capture, or None."""
     if not alg_bytes_per_launch:
         return None
-    h = hashlib.sha256()
-    for f in DECODE_TRAFFIC_SOURCES:
-        with open(os.path.join(ROOT, f), "rb") as fh:
-            h.update(fh.read())
-    if h.hexdigest() != DECODE_TRAFFIC_SHA256:
+    if decode_sources_digest() != DECODE_TRAFFIC_SHA256:
         return None
     return DECODE_TRAFFIC_RATIO * alg_bytes_per_launch
 

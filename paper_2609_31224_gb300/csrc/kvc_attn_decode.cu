@@ -5,15 +5,15 @@
 // resident key (the compacted region, then the live region, the token's own
 // key included).
 //
-// Inside a CTA each warp streams its own pages through a TMA bulk-copy ring in
-// shared memory, computes scores on CUDA cores (packed fp32 FMA), keeps a
-// running max/sum with warp shuffles, and the CTA merges its warps.  Two ways
-// to spread the pages over CTAs (split-K):
+// Inside a CTA each warp streams its own pages through a TMA copy ring in shared
+// memory and computes its scores and P V products, on the tensor cores (mma.sync)
+// for bfloat16 and on CUDA cores (packed fp32 FMA) for binary32, keeping a running
+// max/sum; the CTA then merges its warps.  Two ways to spread the pages over CTAs
+// (split-K):
 //   - stream-K (many sessions): the call's (session, head, page) units are cut
 //     into equal contiguous ranges, one per CTA of 4 warps (three CTAs per SM);
-//   - pair split (few sessions): each (session, head) pair's pages are cut into
-//     k slices, one per CTA of 16 warps (one CTA per SM), so that every page of
-//     the call is in flight at once.
+//   - pair split (fewer sessions): each (session, head) pair's pages are cut into
+//     k slices, one per CTA, so that a call's CTAs fill the GPU in one wave.
 // Either way partial states go to global slots and the last CTA to arrive for a
 // pair merges them (log-sum-exp).  Stream-K publishes them with an acquire-release
 // arrival.  The 16-warp pair split, whose launches are latency-bound, writes each

@@ -1,7 +1,8 @@
 // Device code shared by the two decode translation units (stream-K in
 // kvc_attn_decode.cu, pair split in kvc_attn_decode_split.cu): CTA shapes, the
-// per-warp page pipeline, the CUDA-core page loop, the cross-warp merge and the
-// log-sum-exp merge of split-K partial states.
+// per-warp page pipeline, the page loops (tensor cores for bfloat16, CUDA cores for
+// binary32), the cross-warp merge and the log-sum-exp merge of split-K partial
+// states.
 #pragma once
 
 #include "kvc_launch.cuh"

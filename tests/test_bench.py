@@ -39,15 +39,19 @@ def test_reference_arm_prints_one_json_line():
 def test_traffic_is_reported_only_for_the_captured_sources(tmp_path, monkeypatch):
     import hashlib
     a, b = tmp_path / "a.cu", tmp_path / "b.cuh"
-    a.write_bytes(b"kernel source")
-    b.write_bytes(b"header source")
-    digest = hashlib.sha256(b"kernel source" + b"header source").hexdigest()
+    a.write_text("int kernel(int x) { return x + 1; }  // a comment\n")
+    b.write_text("/* header */ int y;\n")
+    digest = hashlib.sha256(b"int kernel(int x) { return x + 1; }" + b"int y;").hexdigest()
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     monkeypatch.setattr(bench, "DECODE_TRAFFIC_SOURCES", ("a.cu", "b.cuh"))
     monkeypatch.setattr(bench, "DECODE_TRAFFIC_SHA256", digest)
     assert bench.decode_traffic(1000.0) == pytest.approx(1000.0 * bench.DECODE_TRAFFIC_RATIO)
     assert bench.decode_traffic(None) is None
-    a.write_bytes(b"kernel source, changed")
+    # comments and layout do not count ...
+    a.write_text("int kernel(int x)\n{\n  return x + 1;  // another comment\n}\n")
+    assert bench.decode_traffic(1000.0) == pytest.approx(1000.0 * bench.DECODE_TRAFFIC_RATIO)
+    # ... code does
+    a.write_text("int kernel(int x) { return x + 2; }\n")
     assert bench.decode_traffic(1000.0) is None
 
 
