@@ -400,6 +400,29 @@ def test_decode_4warp_tier_at_full_budget():
     assert ls.n_compared >= 10 * 2 + 12 + 16 + 19
 
 
+def test_f32_decode_every_tier():
+    """Binary32 decode in every dispatch tier: 480 sessions of the tiny binary32 shape (one
+    KV head each) starting together, so that a step's decode rounds shrink from 480
+    sessions (stream-K) through the 4-warp pair split with one, two and more slices per
+    pair down to the 16-warp pair split; every output of every decode call of every
+    third step compared with the oracle, every evict bit-exact."""
+    w = S.TINY_F32.with_(n_sessions=480, offset_max=2, budget=64, window=1, seed=7)
+    ls, _ = _lockstep(w, n_units=12)
+    seen = set()
+
+    def select(step, c, i, layer):
+        if c.kind != "decode" or step % 3:
+            return None
+        seen.add(_decode_tier(len(c.sessions), w.kv_heads))
+        return "all"
+
+    for _ in range(len(ls.drv.sched)):
+        ls.run_step(select=select)
+    if _sms() == 152:
+        assert {"streamk", "split4", "split16"} <= seen
+    assert ls.n_compared > 1000
+
+
 def test_decode_4warp_tier_one_and_two_slices():
     """Decode calls of 20-57 sessions, where the 4-warp pair split gives every (session, KV
     head) pair two slices (20-28 sessions, merged by the last to arrive) or one (29-57, no
